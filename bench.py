@@ -1,0 +1,479 @@
+#!/usr/bin/env python
+"""Throughput of the MPM hot path on one GB300 per rank.
+
+A step is one pass of the whole path over one batch of synthetic tokens:
+merge (Algorithm 1) -> merge -> compose maps (Eq. 3) -> gather (Eq. 4).
+Between the two merges a seeded N(0, 0.05^2) perturbation stands in for the
+encoder blocks; it is not part of MPM and is not timed.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload vit_b]
+  python bench.py --impl reference ...   # the fp64 CPU oracle on host cores
+
+Timing: CUDA events on the launch stream bracket the two timed segments of
+every step (merge 1; merge 2 + compose + gather); L2 is flushed by a 256 MiB
+write before every step; W untimed warm-up steps; barrier + synchronize on
+both sides; the max over ranks is reported.  Each rank processes its own
+batch (images are independent: replicas, weak scaling, no collective on the
+data path).  One JSON line is printed by rank 0.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import platform
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "MPM images/sec (merge+compose+unmerge); % bf16 tensor peak, % HBM BW"
+UNIT = "images/s"
+DEFAULT_WORKLOAD = "vit_b"
+PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
+# Fallback denominators when the measured file is absent.
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+L2_FLUSH_BYTES = 256 << 20
+KERNELS_PER_MERGE = 4
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "affinity_tc_traffic.txt")
+
+
+def parse_args():
+    p = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=20)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", choices=["mpm", "reference"], default="mpm")
+    p.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--cpu-seconds", type=float, default=15.0, help="target CPU time of the oracle sample")
+    p.add_argument("--no-e2e", action="store_true")
+    return p.parse_args()
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def load_peaks():
+    try:
+        with open(PEAKS_FILE) as f:
+            pk = json.load(f)
+        return pk, "measured"
+    except (OSError, ValueError):
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+def workload_desc(cfg, batch):
+    sizes = np.diff(batch.offsets)
+    return {
+        "workload": f"{cfg.name}: {cfg.description}",
+        "images": int(cfg.batch),
+        "tokens": int(batch.rows),
+        "tokens_per_image": int(sizes[0]) if len(set(sizes.tolist())) == 1 else "mixed",
+        "dim": int(cfg.dim),
+        "insertions": int(cfg.insertions),
+        "seed": int(cfg.seed),
+        "l2": "flushed by a 256 MiB write before every step",
+        "untimed": "the seeded N(0,0.05^2) stand-in for the encoder blocks between the two merges",
+        "parallelism": "replicas (each rank merges its own batch; no data-path collective)",
+    }
+
+
+# ---------------------------------------------------------------------------
+# The fp64 oracle on the host cores (cpu_baseline leg and --impl reference)
+# ---------------------------------------------------------------------------
+def oracle_image_pipeline(cfg, x_img, b):
+    """merge -> noise -> merge -> compose -> gather for one image (oracle)."""
+    import torch
+
+    import oracle
+    from workloads import DTYPES, apply_noise, stage_noise
+
+    def stored(v):
+        return oracle.round_bf16(v) if cfg.dtype == "bf16" else oracle.round_f32(v).astype(np.float64)
+
+    m1 = oracle.merge_image(x_img)
+    if cfg.insertions == 1:
+        return oracle.gather(stored(m1.x_out), m1.r)
+    s1 = torch.from_numpy(stored(m1.x_out).astype(np.float32)).to(DTYPES[cfg.dtype])
+    noise = stage_noise(cfg.seed, [m1.n_out], cfg.dim, images=[b])
+    s1n = apply_noise(s1, noise).double().numpy()
+    m2 = oracle.merge_image(s1n)
+    r_star = oracle.compose(m1.r, m2.r)
+    return oracle.gather(stored(m2.x_out), r_star)
+
+
+def oracle_sample(cfg, batch, seconds):
+    """Times the oracle on as many images as fit in about `seconds`."""
+    x = batch.tokens.double().numpy()
+    t0 = time.perf_counter()
+    done = 0
+    while done < cfg.batch:
+        b = done
+        oracle_image_pipeline(cfg, x[batch.offsets[b]:batch.offsets[b + 1]], b)
+        done += 1
+        if time.perf_counter() - t0 > seconds:
+            break
+    dt = time.perf_counter() - t0
+    return done, dt
+
+
+def host_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def cpu_baseline_obj(images, seconds, cfg):
+    return {
+        "value": images / seconds,
+        "unit": UNIT,
+        "cores": host_cores(),
+        "kind": "oracle",
+        "sample": (f"{images} of {cfg.batch} images of {cfg.name}, full pipeline per image "
+                   f"(merge, stand-in noise, merge, compose, gather) in fp64 numpy, {seconds:.1f} s wall; "
+                   f"BLAS threads default, {platform.machine()} host"),
+    }
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    from workloads import CONFIGS, make_batch
+
+    cfg = CONFIGS[args.workload]
+    batch = make_batch(cfg)
+    x = batch.tokens.double().numpy()
+    for s in range(args.warmup):
+        b = s % cfg.batch
+        oracle_image_pipeline(cfg, x[batch.offsets[b]:batch.offsets[b + 1]], b)
+    t0 = time.perf_counter()
+    for s in range(args.steps):
+        b = (args.warmup + s) % cfg.batch
+        oracle_image_pipeline(cfg, x[batch.offsets[b]:batch.offsets[b + 1]], b)
+    dt = time.perf_counter() - t0
+    value = args.steps / dt
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": dict(workload_desc(cfg, batch), step="one image of the workload per step"),
+        "impl": "reference",
+        "cpu_baseline": dict(cpu_baseline_obj(args.steps, dt, cfg)),
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ---------------------------------------------------------------------------
+# Clock sampling during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.proc = None
+        self.gpu = gpu_index
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{gpu_index}.csv")
+
+    def start(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.QUERY}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=self.fh, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.fh.close()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    smax.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for name, flag in zip(names, parts[5:9]):
+                    if flag.lower() == "active":
+                        reasons.add(name)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def traffic_for(kernel_file: str):
+    """DRAM bytes per launch from the committed ncu summary, if the kernel is unchanged."""
+    try:
+        with open(TRAFFIC_FILE) as f:
+            fields = dict(line.strip().split("=", 1) for line in f if "=" in line and not line.startswith("#"))
+        with open(kernel_file, "rb") as f:
+            sha = hashlib.sha256(f.read()).hexdigest()[:16]
+        if fields.get("source_sha256_16") == sha:
+            return float(fields["dram_bytes_per_launch"])
+    except (OSError, ValueError, KeyError):
+        pass
+    return None
+
+
+# ---------------------------------------------------------------------------
+# The GPU path
+# ---------------------------------------------------------------------------
+def run_mpm(args):
+    import torch
+    import torch.distributed as dist
+
+    import paper_2604_05718_gb300 as mpm
+    from paper_2604_05718_gb300 import build
+    from workloads import CONFIGS, apply_noise, make_batch, stage_noise
+
+    rank, world, local = dist_env()
+    if not torch.cuda.is_available():
+        raise RuntimeError("bench.py needs a CUDA device")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+    build.build()
+    mpm.library()
+
+    cfg = CONFIGS[args.workload]
+    batch = make_batch(cfg)
+    rows, dim, nimg = batch.rows, cfg.dim, cfg.batch
+    esize = 2 if cfg.dtype == "bf16" else 4
+    stream = torch.cuda.current_stream(dev)
+
+    # CPU baseline first (pure numpy, rank 0, one GPU only), before GPU work.
+    cpu_base = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        n_img, secs = oracle_sample(cfg, batch, args.cpu_seconds)
+        cpu_base = cpu_baseline_obj(n_img, secs, cfg)
+
+    x0 = batch.tokens.to(dev)
+    off0 = torch.from_numpy(batch.offsets).to(dev)
+    ws = mpm.new_workspace(rows, nimg, dim, x0.dtype, dev)
+    x1 = torch.empty_like(x0)
+    off1 = torch.empty(nimg + 1, dtype=torch.int64, device=dev)
+    m1 = torch.empty(rows, dtype=torch.int32, device=dev)
+    x1n = torch.zeros_like(x0)
+    x2 = torch.empty_like(x0)
+    off2 = torch.empty_like(off1)
+    m2 = torch.empty_like(m1)
+    rstar = torch.empty_like(m1)
+    up = torch.empty_like(x0)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+
+    # One untimed pass fixes the stage-1 counts, hence the stand-in noise.
+    mpm.merge(x0, off0, workspace=ws, out_tokens=x1, out_offsets=off1, out_map=m1)
+    off1_h = off1.cpu().numpy()
+    t1 = int(off1_h[-1])
+    two = cfg.insertions == 2
+    noise = stage_noise(cfg.seed, np.diff(off1_h).tolist(), dim).to(dev) if two else None
+
+    def new_events(n):
+        evs = [torch.cuda.Event(enable_timing=True) for _ in range(n)]
+        for e in evs:
+            e.record(stream)  # materialise the CUDA event handles
+        return evs
+
+    class StepEvents:
+        def __init__(self):
+            self.seg = new_events(4)       # [merge1 start, merge1 end, rest start, rest end]
+            self.k1 = new_events(8)        # merge 1 kernels
+            self.k2 = new_events(8)        # merge 2 kernels
+            self.cg = new_events(2)        # between compose and gather
+
+    def step(ev: StepEvents, host_in=None, host_out=None):
+        flush.fill_(1)
+        ev.seg[0].record(stream)
+        if host_in is not None:
+            x0.copy_(host_in[0], non_blocking=True)
+            off0.copy_(host_in[1], non_blocking=True)
+        mpm.merge(x0, off0, workspace=ws, out_tokens=x1, out_offsets=off1, out_map=m1, stage_events=ev.k1)
+        ev.seg[1].record(stream)
+        if two:
+            x1n[:t1] = apply_noise(x1[:t1], noise)
+        ev.seg[2].record(stream)
+        if two:
+            mpm.merge(x1n, off1, workspace=ws, out_tokens=x2, out_offsets=off2, out_map=m2, stage_events=ev.k2)
+            mpm.compose_maps(m1, off0, m2, off1, out=rstar)
+            ev.cg[0].record(stream)
+            mpm.unmerge_gather(x2, off2, rstar, off0, out=up)
+        else:
+            ev.cg[0].record(stream)
+            mpm.unmerge_gather(x1, off1, m1, off0, out=up)
+        ev.cg[1].record(stream)
+        if host_out is not None:
+            host_out.copy_(up, non_blocking=True)
+        ev.seg[3].record(stream)
+
+    def barrier():
+        torch.cuda.synchronize(dev)
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    def max_over_ranks(v: float) -> float:
+        if world == 1:
+            return v
+        t = torch.tensor([v], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    # ---------------- device-resident timed loop ----------------
+    events = [StepEvents() for _ in range(args.steps)]
+    warm = StepEvents()
+    for _ in range(args.warmup):
+        step(warm)
+    assert mpm.device_status(ws) == 0, "device status reported an error during warm-up"
+    clocks = ClockSampler(local)
+    barrier()
+    clocks.start()
+    wall0 = time.perf_counter()
+    for ev in events:
+        step(ev)
+    barrier()
+    wall = time.perf_counter() - wall0
+    clk = clocks.stop()
+    seg_ms = [ev.seg[0].elapsed_time(ev.seg[1]) + ev.seg[2].elapsed_time(ev.seg[3]) for ev in events]
+    ms = max_over_ranks(statistics.mean(seg_ms))
+    off2_h = off2.cpu().numpy() if two else off1_h
+    assert mpm.device_status(ws) == 0, "device status reported an error in the timed loop"
+
+    # Per-kernel durations inside the timed region.
+    def kernel_ms(key, k):
+        return [getattr(ev, key)[2 * k].elapsed_time(getattr(ev, key)[2 * k + 1]) for ev in events]
+
+    names = ["prep", "affinity", "mutual_scan", "pair_average"]
+    kern = {}
+    for k, nm in enumerate(names):
+        kern[f"{nm}_1_us"] = 1e3 * statistics.mean(kernel_ms("k1", k))
+        if two:
+            kern[f"{nm}_2_us"] = 1e3 * statistics.mean(kernel_ms("k2", k))
+    cg = [ev.cg[0].elapsed_time(ev.cg[1]) for ev in events]
+    kern["gather_us"] = 1e3 * statistics.mean(cg)
+
+    peaks, peak_kind = load_peaks()
+    n0 = np.diff(batch.offsets).astype(np.float64)
+    n1 = np.diff(off1_h).astype(np.float64)
+    n2 = np.diff(off2_h).astype(np.float64)
+    flops1 = float(np.sum(2.0 * n0 * n0 * dim))
+    flops2 = float(np.sum(2.0 * n1 * n1 * dim)) if two else 0.0
+    aff_ms = kernel_ms("k1", 1) + (kernel_ms("k2", 1) if two else [])
+    aff_flops = [flops1] * args.steps + ([flops2] * args.steps if two else [])
+    launches = len(aff_ms)
+    achieved_tflops = sum(aff_flops) / (sum(aff_ms) * 1e-3) / 1e12
+    flops_per_launch = sum(aff_flops) / launches
+    tensor_peak = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
+    traffic = traffic_for(os.path.join(ROOT, "paper_2604_05718_gb300", "csrc", "affinity_tc.cu"))
+    roofline = {
+        "kernel": "affinity_tc (fused cosine affinity + arg max, tcgen05)",
+        "bound": "tensor", "achieved": achieved_tflops, "peak": tensor_peak, "unit": "TFLOP/s",
+        "frac": achieved_tflops / tensor_peak,
+        "peak_kind": f"{peak_kind} bf16 sustained (kernel timed inside the step loop)",
+        "flops_per_launch": flops_per_launch,
+        "flops_definition": "Eq. 1 dense S = X X^T: 2 * N_b^2 * D per image per stage",
+        "frac_of_burst_peak": achieved_tflops / peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]),
+        "traffic": traffic,
+    }
+    # HBM fractions of the bandwidth kernels (algorithmic bytes / event time).
+    hbm = peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
+    avg1 = float((n0.sum() + n1.sum()) * dim * esize + 12 * n0.sum())
+    gat = float((n2.sum() + n0.sum()) * dim * esize + 4 * n0.sum())
+    norm1 = float(n0.sum() * dim * esize + 12 * n0.sum())
+    hbm_kernels = {
+        "pair_average_1_gbs": avg1 / (kern["pair_average_1_us"] * 1e-6) / 1e9,
+        "gather_gbs": gat / (kern["gather_us"] * 1e-6) / 1e9,
+        "prep_1_gbs": norm1 / (kern["prep_1_us"] * 1e-6) / 1e9,
+        "peak_gbs": hbm, "peak_kind": f"{peak_kind} copy bandwidth",
+    }
+    for k in ("pair_average_1", "gather", "prep_1"):
+        hbm_kernels[k + "_frac"] = hbm_kernels[k + "_gbs"] / hbm
+
+    # ---------------- end to end: host buffers, copies inside the timed region ----------------
+    e2e = None
+    if not args.no_e2e:
+        host_x = batch.tokens.pin_memory()
+        host_off = torch.from_numpy(batch.offsets).pin_memory()
+        host_up = torch.empty(up.shape, dtype=up.dtype).pin_memory()
+        e_events = [StepEvents() for _ in range(args.steps)]
+        for _ in range(max(1, args.warmup)):
+            step(warm, (host_x, host_off), host_up)
+        barrier()
+        for ev in e_events:
+            step(ev, (host_x, host_off), host_up)
+        barrier()
+        e_ms = max_over_ranks(statistics.mean(
+            [ev.seg[0].elapsed_time(ev.seg[1]) + ev.seg[2].elapsed_time(ev.seg[3]) for ev in e_events]))
+        # The copied-back grid must be the device result.
+        assert torch.equal(host_up.to(dev), up)
+        e2e = {"value": world * nimg / (e_ms * 1e-3), "unit": UNIT,
+               "h2d_bytes_per_step": int(host_x.numel() * host_x.element_size() + host_off.numel() * 8),
+               "d2h_bytes_per_step": int(host_up.numel() * host_up.element_size()),
+               "ms_per_step": e_ms}
+
+    if world > 1:
+        dist.barrier()
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": world * nimg / (ms * 1e-3), "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": cfg.dtype, "data": "synthetic",
+            "config": workload_desc(cfg, batch),
+            "tokens_per_s": world * rows / (ms * 1e-3),
+            "merged_tokens": {"stage0": int(n0.sum()), "stage1": int(n1.sum()), "stage2": int(n2.sum())},
+            "roofline": roofline,
+            "hbm_kernels": hbm_kernels,
+            "kernels_us": kern,
+            "cpu_baseline": cpu_base,
+            "e2e": e2e,
+            "clocks": clk,
+            "gpu_launches": (2 * KERNELS_PER_MERGE + 2 if two else KERNELS_PER_MERGE + 1) * args.steps,
+            "wall_s_timed_loop": wall,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_mpm(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,197 @@
+/*
+ * mpm.h - C ABI of the GB300 (sm_103a) Mutual Pair Merging library.
+ *
+ * Mutual Pair Merging (MPM, arxiv 2604.05718) shortens the image-token
+ * sequence of a ViT: it L2-normalises each image's tokens, takes every
+ * token's cosine nearest neighbour, averages each mutual nearest-neighbour
+ * pair into one token and records an integer merge map (Section 3.2,
+ * Eq. 1-2, Algorithm 1).  Maps of successive insertions are composed
+ * (Eq. 3) and a gather restores the full token grid before the decoder
+ * (Eq. 4).
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - Batches are ragged and packed: image b owns rows [off[b], off[b+1]) of
+ *    a row-major [rows, dim] token matrix.  `offsets` arrays are int64
+ *    [batch + 1] in DEVICE memory with off[0] == 0, non-decreasing values and
+ *    off[batch] <= rows.  Images are independent (Section 3.1); empty images
+ *    and single-token images are legal (a single token is a singleton).
+ *  - `rows` is the number of rows ALLOCATED for a token or map buffer.  It
+ *    bounds every access, so the host never needs to read off[batch].
+ *  - Every pointer is a device pointer owned by the caller; the library
+ *    allocates and frees nothing.  Token buffers must be 16-byte aligned and
+ *    dim must be a multiple of 8 (bf16) or 4 (fp32) so that rows are 16-byte
+ *    aligned; otherwise MPM_ERR_ALIGNMENT.  1 <= dim <= 16384.
+ *  - Merge maps are int32 and LOCAL: map[off[b] + p] is the output row of
+ *    input row p within image b (0-based; Algorithm 1 counts from 1).
+ *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *    stream).  Every call is asynchronous and stream-ordered.  The returned
+ *    status covers host-side validation and launch errors only.
+ *  - Device-side problems (offsets that are not monotone, a map entry out of
+ *    range, a bounded wait that expired) are recorded, first error wins, in a
+ *    device status word: the merge workspace's (read it with
+ *    mpm_get_device_status after synchronising), or the optional
+ *    `device_status` int32 of compose and gather.  Kernels never trap: a bad
+ *    entry is skipped (its output row zeroed, its map entry set to -1).
+ */
+#ifndef MPM_H
+#define MPM_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Only the entry points below are exported from libmpm.so. */
+#if defined(__GNUC__)
+#define MPM_API __attribute__((visibility("default")))
+#else
+#define MPM_API
+#endif
+
+#define MPM_ABI_VERSION 1
+#define MPM_MAX_DIM 16384
+
+typedef enum mpm_dtype {
+  MPM_F32 = 0,  /* IEEE binary32 tokens */
+  MPM_BF16 = 1  /* bfloat16 tokens */
+} mpm_dtype;
+
+typedef enum mpm_status {
+  MPM_OK = 0,
+  MPM_ERR_INVALID_ARG = 1,     /* null pointer, negative size, bad enum */
+  MPM_ERR_UNSUPPORTED = 2,     /* no device of compute capability 10.3, or dim too large */
+  MPM_ERR_ALIGNMENT = 3,       /* token pointer or row size not 16-byte aligned */
+  MPM_ERR_WORKSPACE = 4,       /* workspace missing, too small or misaligned */
+  MPM_ERR_CUDA = 5,            /* a CUDA runtime or driver call failed */
+  MPM_ERR_DEVICE_CHECK = 6,    /* (device status) invalid offsets or map entry */
+  MPM_ERR_DEVICE_TIMEOUT = 7,  /* (device status) a bounded wait expired */
+  MPM_ERR_ALIASING = 8         /* an output buffer overlaps an input buffer */
+} mpm_status;
+
+/* Which kernel computes the nearest neighbours (Eq. 1 + arg max). */
+typedef enum mpm_nn_algo {
+  MPM_NN_AUTO = 0,    /* tensor cores for bf16, CUDA-core fp32 otherwise */
+  MPM_NN_SIMT = 1,    /* CUDA-core fp32 FMA tiles (any dtype) */
+  MPM_NN_TCGEN05 = 2  /* TMA + tcgen05 MMA into TMEM (bf16 only) */
+} mpm_nn_algo;
+
+/* Version of this ABI (MPM_ABI_VERSION). */
+MPM_API int32_t mpm_abi_version(void);
+
+/* Human-readable name of a status code (static string, never NULL). */
+MPM_API const char* mpm_status_string(mpm_status status);
+
+/*
+ * Bytes of device workspace that mpm_merge and mpm_nearest_neighbors need
+ * for `rows` token rows and `batch` images.  Returns 0 for invalid sizes.
+ * The workspace must be 256-byte aligned.  It holds per-row inverse norms,
+ * packed arg-max keys, the representative list, per-image counts, sanitised
+ * offsets, the work plan and the device status word.
+ */
+MPM_API size_t mpm_merge_workspace_size(int64_t rows, int32_t batch, int32_t dim, mpm_dtype dtype);
+
+/*
+ * One MPM call on every image of a packed batch (Algorithm 1; Eq. 1-2).
+ *
+ *   tokens       [rows, dim] input tokens (dtype), image b at rows off[b]..
+ *   offsets      int64 [batch + 1] device offsets of the input images
+ *   out_tokens   [rows, dim] output capacity (dtype).  Image b's N'_b merged
+ *                tokens are written at rows out_offsets[b].. in increasing
+ *                order of their representative (the pair's lower index);
+ *                each is (x_i + x_j) / 2 computed in fp32 and rounded to
+ *                nearest even, or the unchanged token for a singleton.
+ *   out_offsets  int64 [batch + 1] device, written: exclusive scan of N'_b
+ *   out_map      int32 [rows] device, written for rows < off[batch]: the
+ *                local output row r(i) of every input row (Algorithm 1)
+ *   workspace    device scratch of mpm_merge_workspace_size(...) bytes
+ *
+ * The nearest neighbour of token i is the j != i of its image maximising the
+ * cosine (x_i . x_j) / (|x_i| |x_j|), with norms floored at 1e-12 and ties
+ * going to the lowest j; (i, j) merge when each is the other's nearest
+ * neighbour (Section 3.2).  N'_b = N_b - #pairs >= ceil(N_b / 2).
+ * out_tokens must not overlap tokens (MPM_ERR_ALIASING).
+ */
+MPM_API mpm_status mpm_merge(const void* tokens, const int64_t* offsets, int32_t batch,
+                     int64_t rows, int32_t dim, mpm_dtype dtype, void* out_tokens,
+                     int64_t* out_offsets, int32_t* out_map, void* workspace,
+                     size_t workspace_bytes, void* stream);
+
+/*
+ * mpm_merge with per-kernel CUDA events, for profiling.  When stage_events
+ * is not NULL it holds 8 cudaEvent_t handles created by the caller (timing
+ * enabled); stage_events[2k] is recorded on `stream` just before kernel k
+ * and stage_events[2k+1] just after it, for k = 0 row norms and work plan,
+ * 1 affinity + arg max (Eq. 1, Algorithm 1 step 3), 2 mutual check and
+ * left-to-right compaction scan (steps 4-6), 3 pair average (Eq. 2).
+ * Otherwise identical to mpm_merge (which is this call with NULL).
+ */
+MPM_API mpm_status mpm_merge_timed(const void* tokens, const int64_t* offsets, int32_t batch,
+                                   int64_t rows, int32_t dim, mpm_dtype dtype, void* out_tokens,
+                                   int64_t* out_offsets, int32_t* out_map, void* workspace,
+                                   size_t workspace_bytes, void* stream,
+                                   void* const* stage_events);
+
+/*
+ * Map composition across two insertions (Eq. 3): r*(p) = r2(r1(p)).
+ *
+ *   map1      int32 [rows0]: stage-1 map, local to image b of offsets0
+ *   offsets0  int64 [batch + 1]: original images (grid rows)
+ *   map2      int32 [rows1]: stage-2 map, local to image b of offsets1
+ *   offsets1  int64 [batch + 1]: stage-1 output images (stage-2 inputs)
+ *   out_map   int32 [rows0], written for rows < offsets0[batch]
+ *   device_status  optional int32 device word (NULL = not reported); an
+ *             out-of-range map1 entry writes -1 and records
+ *             MPM_ERR_DEVICE_CHECK there.
+ * out_map may alias map1 (in-place) but not map2.
+ */
+MPM_API mpm_status mpm_compose_maps(const int32_t* map1, const int64_t* offsets0, int64_t rows0,
+                            const int32_t* map2, const int64_t* offsets1, int64_t rows1,
+                            int32_t batch, int32_t* out_map, int32_t* device_status,
+                            void* stream);
+
+/*
+ * Gather reconstruction (Eq. 4): out[g0_b + p] = merged[m0_b + map[g0_b + p]],
+ * a pure copy that restores the raster order of the original grid.
+ *
+ *   merged          [merged_rows, dim] merged tokens (dtype)
+ *   merged_offsets  int64 [batch + 1]: images of `merged`
+ *   map             int32 [grid_rows]: composed map, local per image
+ *   grid_offsets    int64 [batch + 1]: images of the original grid
+ *   out             [grid_rows, dim] (dtype), written for rows < grid_offsets[batch]
+ *   device_status   optional int32 device word; an out-of-range map entry
+ *                   zeroes that output row and records MPM_ERR_DEVICE_CHECK.
+ * out must not overlap merged (MPM_ERR_ALIASING).
+ */
+MPM_API mpm_status mpm_unmerge_gather(const void* merged, const int64_t* merged_offsets,
+                              int64_t merged_rows, const int32_t* map,
+                              const int64_t* grid_offsets, int64_t grid_rows, int32_t batch,
+                              int32_t dim, mpm_dtype dtype, void* out,
+                              int32_t* device_status, void* stream);
+
+/*
+ * Nearest neighbours only (Eq. 1 and Algorithm 1 step 3), for testing and
+ * diagnostics.  out_nn int32 [rows]: local index b(i) (-1 for a token alone
+ * in its image); out_score float [rows] (may be NULL): the cosine S_{i,b(i)}
+ * as computed in fp32.  `algo` selects the kernel (MPM_NN_TCGEN05 requires
+ * bf16).  Same workspace as mpm_merge.
+ */
+MPM_API mpm_status mpm_nearest_neighbors(const void* tokens, const int64_t* offsets, int32_t batch,
+                                 int64_t rows, int32_t dim, mpm_dtype dtype,
+                                 mpm_nn_algo algo, int32_t* out_nn, float* out_score,
+                                 void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * Copies the device status word of a merge workspace into *host_code
+ * (synchronous on `stream`) and clears it.  Returns MPM_OK when the copy
+ * worked; *host_code is then MPM_OK or the first device error.
+ */
+MPM_API mpm_status mpm_get_device_status(void* workspace, int32_t* host_code, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MPM_H */

@@ -298,4 +298,4 @@ def round_bf16(x: np.ndarray) -> np.ndarray:
     q = np.ldexp(1.0, np.maximum(e, -125) - 8)
     y = np.rint(x / q) * q
     bf16_max = np.ldexp(255.0, 120)  # (2 - 2^-7) * 2^127
-    return np.where(np.abs(y) > bf16_max, np.sign(x) * np.inf, y)
+    return np.where(np.abs(y) > bf16_max, np.copysign(np.inf, x), y)

@@ -1,0 +1,18 @@
+"""GB300 (sm_103a) Mutual Pair Merging: C-ABI CUDA library + thin binding.
+
+The compute path lives in ``libmpm.so`` (CUDA kernels for sm_103a, built by
+``paper_2604_05718_gb300.build.build()``); ``paper_2604_05718_gb300.mpm``
+marshals torch tensors into its C entry points.
+"""
+
+from .mpm import (  # noqa: F401
+    MPMError,
+    compose_maps,
+    device_status,
+    library,
+    merge,
+    nearest_neighbors,
+    new_workspace,
+    unmerge_gather,
+    workspace_size,
+)

@@ -1,0 +1,178 @@
+// Device helpers shared by the MPM kernels: status reporting, offsets
+// lookup, the packed arg-max key and 16-byte vector arithmetic.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "launch.h"
+
+namespace mpm {
+
+// First error wins; `st` may be null (not reported).
+__device__ __forceinline__ void report(int32_t* st, int32_t code, int32_t detail) {
+  if (st != nullptr && atomicCAS(st, 0, code) == 0) st[1] = detail;
+}
+
+// Index of the image that owns global row g: the largest b < batch with
+// off[b] <= g.  `off` must be non-decreasing (sanitised offsets are).
+__device__ __forceinline__ int find_image(const int64_t* __restrict__ off, int batch, int64_t g) {
+  int lo = 0, hi = batch - 1;
+  while (lo < hi) {
+    int mid = (lo + hi + 1) >> 1;
+    if (__ldg(off + mid) <= g) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
+
+// Same search over the work plan (prefix of work items per image).
+__device__ __forceinline__ int find_item_image(const int64_t* __restrict__ plan, int batch, int64_t w) {
+  int lo = 0, hi = batch - 1;
+  while (lo < hi) {
+    int mid = (lo + hi + 1) >> 1;
+    if (__ldg(plan + mid) <= w) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
+
+// A total order on floats as unsigned integers (larger float -> larger key).
+__device__ __forceinline__ uint32_t order_f32(float f) {
+  uint32_t u = __float_as_uint(f);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ float unorder_f32(uint32_t k) {
+  uint32_t u = (k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k;
+  return __uint_as_float(u);
+}
+
+// Packed arg-max key: the larger score wins, and on equal scores the lower
+// column j wins, so a 64-bit atomicMax merges partial results in any order
+// to the same answer.  -0 is folded into +0 so that equal scores compare
+// equal.  Key 0 means "no candidate" (it is below every real key).
+__device__ __forceinline__ unsigned long long make_key(float s, int32_t j) {
+  if (s == 0.0f) s = 0.0f;
+  return (static_cast<unsigned long long>(order_f32(s)) << 32) |
+         static_cast<unsigned long long>(0xFFFFFFFFu - static_cast<uint32_t>(j));
+}
+__device__ __forceinline__ int32_t key_index(unsigned long long key) {
+  if (key == 0ull) return -1;
+  return static_cast<int32_t>(0xFFFFFFFFu - static_cast<uint32_t>(key & 0xFFFFFFFFull));
+}
+__device__ __forceinline__ float key_score(unsigned long long key) {
+  return unorder_f32(static_cast<uint32_t>(key >> 32));
+}
+
+// ---------------------------------------------------------------------------
+// 16-byte vectors: 8 bf16 or 4 fp32 lanes.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float sumsq16(uint4 v, bool bf16) {
+  float s = 0.f;
+  if (bf16) {
+    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      float2 f = __bfloat1622float2(h[k]);
+      s = fmaf(f.x, f.x, s);
+      s = fmaf(f.y, f.y, s);
+    }
+  } else {
+    const float* f = reinterpret_cast<const float*>(&v);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) s = fmaf(f[k], f[k], s);
+  }
+  return s;
+}
+
+// (a + b) / 2 lane by lane: fp32 add, exact halving, round to nearest even.
+__device__ __forceinline__ uint4 avg16(uint4 a, uint4 b, bool bf16) {
+  uint4 r;
+  if (bf16) {
+    const __nv_bfloat162* ha = reinterpret_cast<const __nv_bfloat162*>(&a);
+    const __nv_bfloat162* hb = reinterpret_cast<const __nv_bfloat162*>(&b);
+    __nv_bfloat162* hr = reinterpret_cast<__nv_bfloat162*>(&r);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      float2 fa = __bfloat1622float2(ha[k]);
+      float2 fb = __bfloat1622float2(hb[k]);
+      hr[k] = __floats2bfloat162_rn((fa.x + fb.x) * 0.5f, (fa.y + fb.y) * 0.5f);
+    }
+  } else {
+    const float* fa = reinterpret_cast<const float*>(&a);
+    const float* fb = reinterpret_cast<const float*>(&b);
+    float* fr = reinterpret_cast<float*>(&r);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) fr[k] = (fa[k] + fb[k]) * 0.5f;
+  }
+  return r;
+}
+
+__device__ __forceinline__ uint4 ld_stream(const uint4* p) { return __ldcs(p); }
+__device__ __forceinline__ void st_stream(uint4* p, uint4 v) { __stcs(p, v); }
+
+// ---------------------------------------------------------------------------
+// Warp / block scans (inclusive), blockDim a multiple of 32, <= 1024.
+// ---------------------------------------------------------------------------
+template <typename T>
+__device__ __forceinline__ T warp_incl_sum(T v) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    T o = __shfl_up_sync(0xFFFFFFFFu, v, d);
+    if (lane >= d) v += o;
+  }
+  return v;
+}
+
+template <typename T>
+__device__ __forceinline__ T warp_incl_max(T v) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    T o = __shfl_up_sync(0xFFFFFFFFu, v, d);
+    if (lane >= d) v = v > o ? v : o;
+  }
+  return v;
+}
+
+// Inclusive block sum scan; returns the block total in *total.  `sh` needs
+// 32 elements of shared memory.  Must be called by all threads.
+template <typename T>
+__device__ __forceinline__ T block_incl_sum(T v, T* sh, T* total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int nwarps = (blockDim.x + 31) >> 5;
+  T x = warp_incl_sum(v);
+  if (lane == 31) sh[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    T w = lane < nwarps ? sh[lane] : T(0);
+    w = warp_incl_sum(w);
+    sh[lane] = w;
+  }
+  __syncthreads();
+  T base = warp > 0 ? sh[warp - 1] : T(0);
+  *total = sh[nwarps - 1];
+  __syncthreads();
+  return x + base;
+}
+
+template <typename T>
+__device__ __forceinline__ T block_incl_max(T v, T* sh, T* total, T lowest) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int nwarps = (blockDim.x + 31) >> 5;
+  T x = warp_incl_max(v);
+  if (lane == 31) sh[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    T w = lane < nwarps ? sh[lane] : lowest;
+    w = warp_incl_max(w);
+    sh[lane] = w;
+  }
+  __syncthreads();
+  T base = warp > 0 ? sh[warp - 1] : lowest;
+  *total = sh[nwarps - 1];
+  __syncthreads();
+  return x > base ? x : base;
+}
+
+}  // namespace mpm

@@ -1,0 +1,347 @@
+// Bandwidth-bound MPM kernels: row norms (Eq. 1), the mutual check and
+// left-to-right representative scan (Algorithm 1 steps 4-6), the pair
+// average with compaction (Eq. 2), map composition (Eq. 3) and the gather
+// reconstruction (Eq. 4).  All token traffic moves in 16-byte vectors, one
+// warp per row; grids are sized from the SM count and loop over rows.
+#include <math.h>
+
+#include "../../include/mpm.h"
+#include "common.cuh"
+
+namespace mpm {
+namespace {
+
+constexpr int kThreads = 256;
+
+__device__ __forceinline__ int64_t clamp64(int64_t v, int64_t lo, int64_t hi) {
+  return v < lo ? lo : (v > hi ? hi : v);
+}
+
+// Finds the image of row p, reusing the previous answer when p is still in
+// the same image (rows are visited in increasing order by each warp).
+struct ImageCursor {
+  int b = 0;
+  int64_t lo = 1, hi = 0;  // empty: forces the first search
+  __device__ __forceinline__ void locate(const int64_t* off, int batch, int64_t p) {
+    if (p >= lo && p < hi) return;
+    b = find_image(off, batch, p);
+    lo = __ldg(off + b);
+    hi = __ldg(off + b + 1);
+  }
+};
+
+// ---------------------------------------------------------------------------
+// Prep: status reset, offsets sanitisation + work plan (block 0), inverse
+// row norms and key reset (all blocks).
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads) prep_kernel(const uint8_t* __restrict__ tokens,
+                                                        const int64_t* __restrict__ offsets,
+                                                        int batch, int64_t rows, int row_bytes,
+                                                        bool bf16, int tile_m, int tile_n,
+                                                        Workspace ws) {
+  if (blockIdx.x == 0) {
+    __shared__ int64_t sh[32];
+    __shared__ int bad;
+    if (threadIdx.x == 0) {
+      ws.status[0] = 0;
+      ws.status[1] = 0;
+      ws.status[2] = 0;
+      bad = -1;
+    }
+    __syncthreads();
+    // soff[b] = min(rows, max_{b' <= b} max(off[b'], 0)): non-decreasing and
+    // in range whatever the caller passed; violations are reported.
+    int64_t carry = 0;
+    for (int base = 0; base <= batch; base += kThreads) {
+      const int idx = base + threadIdx.x;
+      int64_t raw = 0, prev = 0;
+      if (idx <= batch) {
+        raw = offsets[idx];
+        prev = idx > 0 ? offsets[idx - 1] : 0;
+        if ((idx == 0 && raw != 0) || raw < prev || raw > rows) atomicCAS(&bad, -1, idx);
+      }
+      int64_t v = idx <= batch ? clamp64(raw, 0, rows) : 0;
+      int64_t total;
+      int64_t m = block_incl_max<int64_t>(v, sh, &total, 0);
+      m = m > carry ? m : carry;
+      if (idx <= batch) ws.soff[idx] = m;
+      carry = total > carry ? total : carry;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0 && bad >= 0) report(ws.status, MPM_ERR_DEVICE_CHECK, bad);
+    // plan[b] = sum_{b' < b} ceil(N_b'/tile_m) * ceil(N_b'/tile_n).
+    __threadfence_block();
+    int64_t acc = 0;
+    for (int base = 0; base <= batch; base += kThreads) {
+      const int idx = base + threadIdx.x;
+      int64_t items = 0;
+      if (idx < batch) {
+        const int64_t n = ws.soff[idx + 1] - ws.soff[idx];
+        items = ((n + tile_m - 1) / tile_m) * ((n + tile_n - 1) / tile_n);
+      }
+      int64_t total;
+      const int64_t incl = block_incl_sum<int64_t>(items, sh, &total);
+      if (idx <= batch) ws.plan[idx] = acc + incl - items;
+      acc += total;
+    }
+  }
+
+  // Inverse norms of every used row, and the arg-max keys reset to "none".
+  const int64_t used = clamp64(offsets[batch], 0, rows);
+  const int lane = threadIdx.x & 31;
+  const int64_t warp = (static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x) >> 5;
+  const int64_t nwarps = (static_cast<int64_t>(gridDim.x) * kThreads) >> 5;
+  const int nvec = row_bytes >> 4;
+  for (int64_t g = warp; g < used; g += nwarps) {
+    const uint4* src = reinterpret_cast<const uint4*>(tokens + g * row_bytes);
+    float s = 0.f;
+    for (int v = lane; v < nvec; v += 32) s += sumsq16(__ldg(src + v), bf16);
+#pragma unroll
+    for (int d = 16; d > 0; d >>= 1) s += __shfl_xor_sync(0xFFFFFFFFu, s, d);
+    if (lane == 0) {
+      ws.inv_norm[g] = 1.0f / fmaxf(sqrtf(s), 1e-12f);
+      ws.keys[g] = 0ull;
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Mutual check + left-to-right representative scan, one block per image.
+// The last block to finish turns the per-image counts into out_offsets.
+// ---------------------------------------------------------------------------
+constexpr int kScanThreads = 1024;
+
+__global__ void __launch_bounds__(kScanThreads) mutual_compact_kernel(int batch, Workspace ws,
+                                                                      int32_t* __restrict__ out_map,
+                                                                      int64_t* __restrict__ out_offsets) {
+  __shared__ int32_t sh[32];
+  __shared__ int64_t sh64[32];
+  __shared__ int is_last;
+  const int b = blockIdx.x;
+  const int64_t base = ws.soff[b];
+  const int n = static_cast<int>(ws.soff[b + 1] - base);
+  int carry = 0;
+  for (int c0 = 0; c0 < n; c0 += kScanThreads) {
+    const int i = c0 + threadIdx.x;
+    int rep = 0, partner = -1;
+    if (i < n) {
+      int j = key_index(ws.keys[base + i]);
+      if (j >= n || j == i || (j < 0 && n > 1)) {
+        report(ws.status, MPM_ERR_DEVICE_CHECK, static_cast<int32_t>(base + i));
+        j = -1;
+      }
+      // (i, j) is a pair of P when b(j) = i as well (Section 3.2).
+      if (j >= 0 && key_index(ws.keys[base + j]) == i) partner = j;
+      rep = (partner < 0 || i < partner) ? 1 : 0;
+    }
+    int total;
+    const int incl = block_incl_sum<int>(rep, sh, &total);
+    if (rep) {
+      const int r = carry + incl - 1;
+      out_map[base + i] = r;
+      if (partner > i) out_map[base + partner] = r;
+      ws.reps[base + r] = make_int2(i, partner);
+    }
+    carry += total;
+  }
+  if (threadIdx.x == 0) {
+    ws.count[b] = carry;
+    __threadfence();
+    const int prev = atomicAdd(reinterpret_cast<int*>(&ws.status[2]), 1);
+    is_last = (prev == batch - 1);
+  }
+  __syncthreads();
+  if (!is_last) return;
+  __threadfence();
+  int64_t acc = 0;
+  for (int c0 = 0; c0 <= batch; c0 += kScanThreads) {
+    const int idx = c0 + threadIdx.x;
+    const int64_t v = idx < batch ? static_cast<int64_t>(__ldcg(ws.count + idx)) : 0;
+    int64_t total;
+    const int64_t incl = block_incl_sum<int64_t>(v, sh64, &total);
+    if (idx <= batch) out_offsets[idx] = acc + incl - v;
+    acc += total;
+  }
+  if (threadIdx.x == 0) ws.status[2] = 0;
+}
+
+// ---------------------------------------------------------------------------
+// Pair average + compaction (Eq. 2): one warp per output row.
+// ---------------------------------------------------------------------------
+template <int U>
+__global__ void __launch_bounds__(kThreads) pair_average_kernel(const uint8_t* __restrict__ tokens,
+                                                                uint8_t* __restrict__ out,
+                                                                int batch, int64_t rows, int row_bytes,
+                                                                bool bf16, Workspace ws,
+                                                                const int64_t* __restrict__ out_offsets) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warp = (static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x) >> 5;
+  const int64_t nwarps = (static_cast<int64_t>(gridDim.x) * kThreads) >> 5;
+  const int64_t total = clamp64(out_offsets[batch], 0, rows);
+  const int nvec = row_bytes >> 4;
+  ImageCursor cur;
+  for (int64_t t = warp; t < total; t += nwarps) {
+    cur.locate(out_offsets, batch, t);
+    const int64_t in_base = ws.soff[cur.b];
+    const int2 rep = ws.reps[in_base + (t - cur.lo)];
+    const uint4* a = reinterpret_cast<const uint4*>(tokens + (in_base + rep.x) * row_bytes);
+    const uint4* p = reinterpret_cast<const uint4*>(tokens + (in_base + (rep.y >= 0 ? rep.y : rep.x)) * row_bytes);
+    uint4* dst = reinterpret_cast<uint4*>(out + t * row_bytes);
+    for (int v0 = lane; v0 < nvec; v0 += 32 * U) {
+      uint4 va[U], vb[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int v = v0 + 32 * u;
+        if (v < nvec) {
+          va[u] = __ldcs(a + v);
+          vb[u] = rep.y >= 0 ? __ldcs(p + v) : va[u];
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int v = v0 + 32 * u;
+        if (v < nvec) dst[v] = rep.y >= 0 ? avg16(va[u], vb[u], bf16) : va[u];
+      }
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Keys -> nearest neighbour and cosine (test / diagnostics hook).
+// ---------------------------------------------------------------------------
+__global__ void decode_nn_kernel(int batch, int64_t rows, Workspace ws, int32_t* __restrict__ nn,
+                                 float* __restrict__ score) {
+  const int64_t used = ws.soff[batch];
+  for (int64_t g = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; g < used;
+       g += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const unsigned long long k = ws.keys[g];
+    nn[g] = key_index(k);
+    if (score != nullptr) score[g] = k == 0ull ? -INFINITY : key_score(k) * ws.inv_norm[g];
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Map composition (Eq. 3).
+// ---------------------------------------------------------------------------
+// map1 may alias out (in-place composition): each thread reads map1[p]
+// before writing out[p], and no other thread touches row p.
+__global__ void compose_kernel(const int32_t* map1, const int64_t* __restrict__ off0,
+                               int64_t rows0, const int32_t* __restrict__ map2,
+                               const int64_t* __restrict__ off1, int64_t rows1, int batch,
+                               int32_t* out, int32_t* status) {
+  const int64_t used = clamp64(off0[batch], 0, rows0);
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t p = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; p < used; p += stride) {
+    const int b = find_image(off0, batch, p);
+    const int64_t lo0 = __ldg(off0 + b), hi0 = __ldg(off0 + b + 1);
+    const int64_t lo1 = __ldg(off1 + b), hi1 = __ldg(off1 + b + 1);
+    const int32_t m1 = map1[p];
+    int32_t r = -1;
+    if (p >= lo0 && p < hi0 && m1 >= 0 && m1 < hi1 - lo1 && lo1 >= 0 && lo1 + m1 < rows1) {
+      r = __ldg(map2 + lo1 + m1);
+    } else {
+      report(status, MPM_ERR_DEVICE_CHECK, static_cast<int32_t>(p));
+    }
+    out[p] = r;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Gather reconstruction (Eq. 4): one warp per grid row, pure copy.
+// ---------------------------------------------------------------------------
+template <int U>
+__global__ void __launch_bounds__(kThreads) gather_kernel(const uint8_t* __restrict__ merged,
+                                                          const int64_t* __restrict__ moff,
+                                                          int64_t merged_rows,
+                                                          const int32_t* __restrict__ map,
+                                                          const int64_t* __restrict__ goff,
+                                                          int64_t grid_rows, int batch, int row_bytes,
+                                                          uint8_t* __restrict__ out, int32_t* status) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warp = (static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x) >> 5;
+  const int64_t nwarps = (static_cast<int64_t>(gridDim.x) * kThreads) >> 5;
+  const int64_t used = clamp64(goff[batch], 0, grid_rows);
+  const int nvec = row_bytes >> 4;
+  ImageCursor cur;
+  for (int64_t p = warp; p < used; p += nwarps) {
+    cur.locate(goff, batch, p);
+    const int64_t mlo = __ldg(moff + cur.b), mhi = __ldg(moff + cur.b + 1);
+    const int32_t m = __ldg(map + p);
+    const bool ok = p >= cur.lo && p < cur.hi && m >= 0 && m < mhi - mlo && mlo >= 0 &&
+                    mlo + m < merged_rows;
+    if (!ok && lane == 0) report(status, MPM_ERR_DEVICE_CHECK, static_cast<int32_t>(p));
+    const uint4* src = reinterpret_cast<const uint4*>(merged + (ok ? (mlo + m) : 0) * row_bytes);
+    uint4* dst = reinterpret_cast<uint4*>(out + p * row_bytes);
+    for (int v0 = lane; v0 < nvec; v0 += 32 * U) {
+      uint4 val[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int v = v0 + 32 * u;
+        if (v < nvec) val[u] = ok ? __ldg(src + v) : make_uint4(0, 0, 0, 0);
+      }
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int v = v0 + 32 * u;
+        if (v < nvec) __stcs(dst + v, val[u]);
+      }
+    }
+  }
+}
+
+int grid_for(int num_sms, int per_sm) { return (num_sms > 0 ? num_sms : 1) * per_sm; }
+
+}  // namespace
+
+cudaError_t launch_prep(const void* tokens, const int64_t* offsets, int batch, int64_t rows, int dim,
+                        bool bf16, AffinityTile tile, const Workspace& ws, int num_sms,
+                        cudaStream_t stream) {
+  const int row_bytes = dim * (bf16 ? 2 : 4);
+  prep_kernel<<<grid_for(num_sms, 8), kThreads, 0, stream>>>(
+      static_cast<const uint8_t*>(tokens), offsets, batch, rows, row_bytes, bf16, tile.rows,
+      tile.cols, ws);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_mutual_compact(int batch, const Workspace& ws, int32_t* out_map,
+                                  int64_t* out_offsets, cudaStream_t stream) {
+  mutual_compact_kernel<<<batch, kScanThreads, 0, stream>>>(batch, ws, out_map, out_offsets);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_pair_average(const void* tokens, void* out_tokens, int batch, int64_t rows,
+                                int dim, bool bf16, const Workspace& ws,
+                                const int64_t* out_offsets, int num_sms, cudaStream_t stream) {
+  const int row_bytes = dim * (bf16 ? 2 : 4);
+  pair_average_kernel<4><<<grid_for(num_sms, 8), kThreads, 0, stream>>>(
+      static_cast<const uint8_t*>(tokens), static_cast<uint8_t*>(out_tokens), batch, rows,
+      row_bytes, bf16, ws, out_offsets);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_decode_nn(int batch, int64_t rows, const Workspace& ws, int32_t* out_nn,
+                             float* out_score, int num_sms, cudaStream_t stream) {
+  (void)rows;
+  decode_nn_kernel<<<grid_for(num_sms, 4), kThreads, 0, stream>>>(batch, rows, ws, out_nn, out_score);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_compose(const int32_t* map1, const int64_t* off0, int64_t rows0,
+                           const int32_t* map2, const int64_t* off1, int64_t rows1, int batch,
+                           int32_t* out, int32_t* status, int num_sms, cudaStream_t stream) {
+  compose_kernel<<<grid_for(num_sms, 4), kThreads, 0, stream>>>(map1, off0, rows0, map2, off1,
+                                                                  rows1, batch, out, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather(const void* merged, const int64_t* moff, int64_t merged_rows,
+                          const int32_t* map, const int64_t* goff, int64_t grid_rows, int batch,
+                          int dim, bool bf16, void* out, int32_t* status, int num_sms,
+                          cudaStream_t stream) {
+  const int row_bytes = dim * (bf16 ? 2 : 4);
+  gather_kernel<4><<<grid_for(num_sms, 8), kThreads, 0, stream>>>(
+      static_cast<const uint8_t*>(merged), moff, merged_rows, map, goff, grid_rows, batch,
+      row_bytes, static_cast<uint8_t*>(out), status);
+  return cudaGetLastError();
+}
+
+}  // namespace mpm

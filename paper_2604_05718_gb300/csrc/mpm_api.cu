@@ -1,0 +1,261 @@
+// Host side of the MPM C ABI: argument validation, workspace carving and
+// the launch sequence of each entry point.  No allocation happens here:
+// every buffer, including the scratch workspace, belongs to the caller.
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <atomic>
+
+#include "../../include/mpm.h"
+#include "launch.h"
+
+namespace {
+
+using mpm::Workspace;
+
+constexpr size_t kAlign = 256;
+
+size_t round_up(size_t v) { return (v + kAlign - 1) / kAlign * kAlign; }
+
+int elem_size(mpm_dtype dt) { return dt == MPM_BF16 ? 2 : 4; }
+
+bool valid_dtype(mpm_dtype dt) { return dt == MPM_F32 || dt == MPM_BF16; }
+
+struct Layout {
+  size_t status, soff, plan, count, inv_norm, keys, reps, total;
+};
+
+Layout layout(int64_t rows, int32_t batch) {
+  Layout l{};
+  size_t off = 0;
+  l.status = off;
+  off += round_up(sizeof(int32_t) * mpm::kStatusWords);
+  l.soff = off;
+  off += round_up(sizeof(int64_t) * (static_cast<size_t>(batch) + 1));
+  l.plan = off;
+  off += round_up(sizeof(int64_t) * (static_cast<size_t>(batch) + 1));
+  l.count = off;
+  off += round_up(sizeof(int32_t) * static_cast<size_t>(batch));
+  l.inv_norm = off;
+  off += round_up(sizeof(float) * static_cast<size_t>(rows));
+  l.keys = off;
+  off += round_up(sizeof(unsigned long long) * static_cast<size_t>(rows));
+  l.reps = off;
+  off += round_up(sizeof(int2) * static_cast<size_t>(rows));
+  l.total = off;
+  return l;
+}
+
+Workspace carve(void* base, int64_t rows, int32_t batch) {
+  const Layout l = layout(rows, batch);
+  uint8_t* p = static_cast<uint8_t*>(base);
+  Workspace ws;
+  ws.status = reinterpret_cast<int32_t*>(p + l.status);
+  ws.soff = reinterpret_cast<int64_t*>(p + l.soff);
+  ws.plan = reinterpret_cast<int64_t*>(p + l.plan);
+  ws.count = reinterpret_cast<int32_t*>(p + l.count);
+  ws.inv_norm = reinterpret_cast<float*>(p + l.inv_norm);
+  ws.keys = reinterpret_cast<unsigned long long*>(p + l.keys);
+  ws.reps = reinterpret_cast<int2*>(p + l.reps);
+  return ws;
+}
+
+bool sizes_ok(int64_t rows, int32_t batch) {
+  return batch >= 1 && rows >= 0 && rows <= INT32_MAX;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+bool overlap(const void* a, size_t an, const void* b, size_t bn) {
+  const uintptr_t a0 = reinterpret_cast<uintptr_t>(a), b0 = reinterpret_cast<uintptr_t>(b);
+  return an > 0 && bn > 0 && a0 < b0 + bn && b0 < a0 + an;
+}
+
+// SM count of the current device (cached per device).
+int num_sms() {
+  static std::atomic<int> cache[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  const int slot = dev & 63;
+  int v = cache[slot].load();
+  if (v > 0) return v;
+  if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || v <= 0) return 0;
+  cache[slot].store(v);
+  return v;
+}
+
+mpm_status cuda_status(cudaError_t e) { return e == cudaSuccess ? MPM_OK : MPM_ERR_CUDA; }
+
+// Shared validation of the token-matrix arguments.
+mpm_status check_tokens(const void* tokens, int64_t rows, int32_t dim, mpm_dtype dtype) {
+  if (!valid_dtype(dtype) || dim < 1) return MPM_ERR_INVALID_ARG;
+  if (dim > MPM_MAX_DIM) return MPM_ERR_UNSUPPORTED;
+  if (tokens == nullptr && rows > 0) return MPM_ERR_INVALID_ARG;
+  if (!aligned16(tokens) || (static_cast<int64_t>(dim) * elem_size(dtype)) % 16 != 0) return MPM_ERR_ALIGNMENT;
+  return MPM_OK;
+}
+
+// The affinity + arg max stage shared by mpm_merge and mpm_nearest_neighbors.
+mpm_status run_affinity(const void* tokens, const int64_t* offsets, int32_t batch, int64_t rows, int32_t dim,
+                        mpm_dtype dtype, mpm_nn_algo algo, const Workspace& ws, cudaStream_t stream) {
+  const bool bf16 = dtype == MPM_BF16;
+  if (algo == MPM_NN_AUTO) algo = bf16 ? MPM_NN_TCGEN05 : MPM_NN_SIMT;
+  if (algo == MPM_NN_TCGEN05 && !bf16) return MPM_ERR_UNSUPPORTED;
+  if (algo != MPM_NN_SIMT && algo != MPM_NN_TCGEN05) return MPM_ERR_INVALID_ARG;
+  if (algo == MPM_NN_TCGEN05 && !mpm::tc_available()) return MPM_ERR_UNSUPPORTED;
+  const int sms = num_sms();
+  if (sms <= 0) return MPM_ERR_CUDA;
+  const mpm::AffinityTile tile = algo == MPM_NN_TCGEN05 ? mpm::tc_tile() : mpm::simt_tile();
+  cudaError_t e = mpm::launch_prep(tokens, offsets, batch, rows, dim, bf16, tile, ws, sms, stream);
+  if (e != cudaSuccess) return MPM_ERR_CUDA;
+  if (rows == 0) return MPM_OK;  // every image is empty: nothing to compare
+  if (algo == MPM_NN_TCGEN05) {
+    e = mpm::launch_affinity_tc(tokens, batch, rows, dim, ws, sms, stream);
+  } else {
+    e = mpm::launch_affinity_simt(tokens, batch, dim, bf16, ws, sms, stream);
+  }
+  return cuda_status(e);
+}
+
+}  // namespace
+
+extern "C" {
+
+int32_t mpm_abi_version(void) { return MPM_ABI_VERSION; }
+
+const char* mpm_status_string(mpm_status status) {
+  switch (status) {
+    case MPM_OK: return "ok";
+    case MPM_ERR_INVALID_ARG: return "invalid argument";
+    case MPM_ERR_UNSUPPORTED: return "unsupported configuration";
+    case MPM_ERR_ALIGNMENT: return "token buffer or row size not 16-byte aligned";
+    case MPM_ERR_WORKSPACE: return "workspace missing, too small or misaligned";
+    case MPM_ERR_CUDA: return "CUDA error";
+    case MPM_ERR_DEVICE_CHECK: return "device check failed (offsets or map out of range)";
+    case MPM_ERR_DEVICE_TIMEOUT: return "device wait timed out";
+    case MPM_ERR_ALIASING: return "output overlaps input";
+  }
+  return "unknown status";
+}
+
+size_t mpm_merge_workspace_size(int64_t rows, int32_t batch, int32_t dim, mpm_dtype dtype) {
+  if (!sizes_ok(rows, batch) || dim < 1 || !valid_dtype(dtype)) return 0;
+  return layout(rows, batch).total;
+}
+
+mpm_status mpm_nearest_neighbors(const void* tokens, const int64_t* offsets, int32_t batch, int64_t rows,
+                                 int32_t dim, mpm_dtype dtype, mpm_nn_algo algo, int32_t* out_nn,
+                                 float* out_score, void* workspace, size_t workspace_bytes, void* stream) {
+  if (!sizes_ok(rows, batch) || offsets == nullptr || out_nn == nullptr) return MPM_ERR_INVALID_ARG;
+  mpm_status st = check_tokens(tokens, rows, dim, dtype);
+  if (st != MPM_OK) return st;
+  if (workspace == nullptr || (reinterpret_cast<uintptr_t>(workspace) % kAlign) != 0 ||
+      workspace_bytes < layout(rows, batch).total)
+    return MPM_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const Workspace ws = carve(workspace, rows, batch);
+  st = run_affinity(tokens, offsets, batch, rows, dim, dtype, algo, ws, s);
+  if (st != MPM_OK) return st;
+  return cuda_status(mpm::launch_decode_nn(batch, rows, ws, out_nn, out_score, num_sms(), s));
+}
+
+mpm_status mpm_merge_timed(const void* tokens, const int64_t* offsets, int32_t batch, int64_t rows,
+                           int32_t dim, mpm_dtype dtype, void* out_tokens, int64_t* out_offsets,
+                           int32_t* out_map, void* workspace, size_t workspace_bytes, void* stream,
+                           void* const* stage_events) {
+  if (!sizes_ok(rows, batch) || offsets == nullptr || out_offsets == nullptr) return MPM_ERR_INVALID_ARG;
+  if (rows > 0 && (out_tokens == nullptr || out_map == nullptr)) return MPM_ERR_INVALID_ARG;
+  mpm_status st = check_tokens(tokens, rows, dim, dtype);
+  if (st != MPM_OK) return st;
+  if (!aligned16(out_tokens)) return MPM_ERR_ALIGNMENT;
+  const size_t bytes = static_cast<size_t>(rows) * dim * elem_size(dtype);
+  if (overlap(tokens, bytes, out_tokens, bytes)) return MPM_ERR_ALIASING;
+  if (workspace == nullptr || (reinterpret_cast<uintptr_t>(workspace) % kAlign) != 0 ||
+      workspace_bytes < layout(rows, batch).total)
+    return MPM_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const Workspace ws = carve(workspace, rows, batch);
+  const bool bf16 = dtype == MPM_BF16;
+  const mpm_nn_algo algo = bf16 ? MPM_NN_TCGEN05 : MPM_NN_SIMT;
+  if (algo == MPM_NN_TCGEN05 && !mpm::tc_available()) return MPM_ERR_UNSUPPORTED;
+  const int sms = num_sms();
+  if (sms <= 0) return MPM_ERR_CUDA;
+  // Records stage_events[idx] (if profiling) on the launch stream.
+  auto mark = [&](int idx) -> bool {
+    if (stage_events == nullptr) return true;
+    return cudaEventRecord(static_cast<cudaEvent_t>(stage_events[idx]), s) == cudaSuccess;
+  };
+  const mpm::AffinityTile tile = algo == MPM_NN_TCGEN05 ? mpm::tc_tile() : mpm::simt_tile();
+  cudaError_t e = cudaSuccess;
+  if (!mark(0)) return MPM_ERR_CUDA;
+  e = mpm::launch_prep(tokens, offsets, batch, rows, dim, bf16, tile, ws, sms, s);
+  if (e != cudaSuccess || !mark(1) || !mark(2)) return MPM_ERR_CUDA;
+  if (rows > 0) {
+    e = algo == MPM_NN_TCGEN05 ? mpm::launch_affinity_tc(tokens, batch, rows, dim, ws, sms, s)
+                               : mpm::launch_affinity_simt(tokens, batch, dim, bf16, ws, sms, s);
+    if (e != cudaSuccess) return MPM_ERR_CUDA;
+  }
+  if (!mark(3) || !mark(4)) return MPM_ERR_CUDA;
+  e = mpm::launch_mutual_compact(batch, ws, out_map, out_offsets, s);
+  if (e != cudaSuccess || !mark(5) || !mark(6)) return MPM_ERR_CUDA;
+  if (rows > 0) {
+    e = mpm::launch_pair_average(tokens, out_tokens, batch, rows, dim, bf16, ws, out_offsets, sms, s);
+    if (e != cudaSuccess) return MPM_ERR_CUDA;
+  }
+  return mark(7) ? MPM_OK : MPM_ERR_CUDA;
+}
+
+mpm_status mpm_merge(const void* tokens, const int64_t* offsets, int32_t batch, int64_t rows, int32_t dim,
+                     mpm_dtype dtype, void* out_tokens, int64_t* out_offsets, int32_t* out_map, void* workspace,
+                     size_t workspace_bytes, void* stream) {
+  return mpm_merge_timed(tokens, offsets, batch, rows, dim, dtype, out_tokens, out_offsets, out_map, workspace,
+                         workspace_bytes, stream, nullptr);
+}
+
+mpm_status mpm_compose_maps(const int32_t* map1, const int64_t* offsets0, int64_t rows0, const int32_t* map2,
+                            const int64_t* offsets1, int64_t rows1, int32_t batch, int32_t* out_map,
+                            int32_t* device_status, void* stream) {
+  if (!sizes_ok(rows0, batch) || !sizes_ok(rows1, batch) || offsets0 == nullptr || offsets1 == nullptr)
+    return MPM_ERR_INVALID_ARG;
+  if (rows0 == 0) return MPM_OK;
+  if (map1 == nullptr || out_map == nullptr || (map2 == nullptr && rows1 > 0)) return MPM_ERR_INVALID_ARG;
+  if (overlap(out_map, sizeof(int32_t) * rows0, map2, sizeof(int32_t) * rows1)) return MPM_ERR_ALIASING;
+  const int sms = num_sms();
+  if (sms <= 0) return MPM_ERR_CUDA;
+  return cuda_status(mpm::launch_compose(map1, offsets0, rows0, map2, offsets1, rows1, batch, out_map,
+                                         device_status, sms, static_cast<cudaStream_t>(stream)));
+}
+
+mpm_status mpm_unmerge_gather(const void* merged, const int64_t* merged_offsets, int64_t merged_rows,
+                              const int32_t* map, const int64_t* grid_offsets, int64_t grid_rows, int32_t batch,
+                              int32_t dim, mpm_dtype dtype, void* out, int32_t* device_status, void* stream) {
+  if (!sizes_ok(merged_rows, batch) || !sizes_ok(grid_rows, batch) || merged_offsets == nullptr ||
+      grid_offsets == nullptr)
+    return MPM_ERR_INVALID_ARG;
+  mpm_status st = check_tokens(merged, merged_rows, dim, dtype);
+  if (st != MPM_OK) return st;
+  if (grid_rows == 0) return MPM_OK;
+  if (map == nullptr || out == nullptr) return MPM_ERR_INVALID_ARG;
+  if (!aligned16(out)) return MPM_ERR_ALIGNMENT;
+  const size_t row_bytes = static_cast<size_t>(dim) * elem_size(dtype);
+  if (overlap(merged, row_bytes * merged_rows, out, row_bytes * grid_rows)) return MPM_ERR_ALIASING;
+  const int sms = num_sms();
+  if (sms <= 0) return MPM_ERR_CUDA;
+  return cuda_status(mpm::launch_gather(merged, merged_offsets, merged_rows, map, grid_offsets, grid_rows, batch,
+                                        dim, dtype == MPM_BF16, out, device_status, sms,
+                                        static_cast<cudaStream_t>(stream)));
+}
+
+mpm_status mpm_get_device_status(void* workspace, int32_t* host_code, void* stream) {
+  if (workspace == nullptr || host_code == nullptr) return MPM_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int32_t* status = static_cast<int32_t*>(workspace);  // the status word leads the workspace
+  int32_t word[2] = {0, 0};
+  if (cudaMemcpyAsync(word, status, sizeof(word), cudaMemcpyDeviceToHost, s) != cudaSuccess) return MPM_ERR_CUDA;
+  if (cudaStreamSynchronize(s) != cudaSuccess) return MPM_ERR_CUDA;
+  if (cudaMemsetAsync(status, 0, sizeof(word), s) != cudaSuccess) return MPM_ERR_CUDA;
+  *host_code = word[0];
+  return MPM_OK;
+}
+
+}  // extern "C"
