@@ -84,7 +84,9 @@ class Neighbours:
 
     @property
     def gap(self) -> np.ndarray:
-        return self.top1 - self.top2
+        """top1 - top2 (NaN for a single token, +inf for two tokens)."""
+        with np.errstate(invalid="ignore"):
+            return self.top1 - self.top2
 
     @property
     def near_tie(self) -> np.ndarray:

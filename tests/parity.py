@@ -8,8 +8,12 @@ Acceptance (the reading of the paper's determinism statement used here):
   * where the GPU's nearest neighbours equal the oracle's on a whole image,
     the merge map, the merged-token count and the merged features must equal
     the oracle's exactly (features: the oracle's fp64 average rounded once to
-    the storage dtype); the benchmark spec's tolerances (per row, max |gpu - oracle|
-    <= tol * max |oracle row|, tol = 1e-5 fp32, 2e-3 bf16) are checked too;
+    the storage dtype);
+  * the feature tolerances (per row, max |gpu - oracle| <= tol * max |oracle
+    row|, tol = 1e-5 for fp32 and 2e-3 for bf16) compare against the oracle's
+    value in the storage dtype: rounding an exact average to bf16 alone moves
+    it by up to 2^-8 = 3.9e-3 relative, more than the bf16 bound, so the bound
+    can only hold between values stored at the same precision;
   * where a near tie made the GPU pick differently, its result must still be
     the valid left-to-right compaction of mutual pairs of its own neighbours,
     with each merged token the mean of its members.
@@ -123,14 +127,14 @@ def check_image(x: np.ndarray, nn_g: np.ndarray, map_g: np.ndarray, out_g: np.nd
         assert np.array_equal(map_g, res.r), f"{what}: merge map differs from the oracle"
         assert out_g.shape[0] == res.n_out, f"{what}: merged count {out_g.shape[0]} vs {res.n_out}"
         want = round_to(dtype, res.x_out)
-        check_rowwise_tolerance(out_g, res.x_out, tol, what)
+        check_rowwise_tolerance(out_g, want, tol, what)
         assert np.array_equal(out_g, want), f"{what}: merged features not the correctly rounded averages"
         st.images_exact = 1
         return st, res, True
     members = check_partition(nn_g, map_g, n, what)
     assert out_g.shape[0] == len(members)
     mean = np.stack([x[m].mean(axis=0) for m in members])
-    check_rowwise_tolerance(out_g, mean, tol, what)
+    check_rowwise_tolerance(out_g, round_to(dtype, mean), tol, what)
     st.notes.append(f"{what}: {st.nn_deviations} near-tie rows resolved differently (valid)")
     return st, res, False
 
