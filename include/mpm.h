@@ -135,6 +135,34 @@ MPM_API mpm_status mpm_merge_timed(const void* tokens, const int64_t* offsets, i
                                    void* const* stage_events);
 
 /*
+ * mpm_merge for callers that cannot allocate device memory.  The paper has
+ * no counterpart: this is a deployment convenience.  Some callers must not
+ * call cudaMalloc, for example a plug-in inside a framework that has
+ * reserved the whole device memory pool, or a latency-critical loop where
+ * allocation (which can block and synchronise the device) is banned.  This
+ * entry point computes exactly what mpm_merge computes, with the same
+ * arguments minus the workspace: its scratch is a fixed array of
+ * MPM_NO_ALLOC_SCRATCH_BYTES inside the library, one per device, held until
+ * the process exits.
+ *  - Limit: it returns MPM_ERR_WORKSPACE when
+ *    mpm_merge_workspace_size(rows, batch, dim, dtype) exceeds
+ *    MPM_NO_ALLOC_SCRATCH_BYTES (8 MiB: about 400,000 rows at up to 1024
+ *    images), and allocates nothing in any case.
+ *  - The first call on each device looks up the array's device address
+ *    (cudaGetSymbolAddress, which can load the module); make that first call
+ *    before any stream capture on that device.
+ *  - All calls on a device share the one array: calls that overlap on the
+ *    GPU (different streams or host threads) race and must be serialised by
+ *    the caller.  The array keeps the last call's contents; each call clears
+ *    the part that must start at zero.  The device status word lives in the
+ *    shared array and is not readable through mpm_get_device_status.
+ */
+#define MPM_NO_ALLOC_SCRATCH_BYTES (8u << 20)
+MPM_API mpm_status mpm_merge_no_alloc(const void* tokens, const int64_t* offsets, int32_t batch,
+                                      int64_t rows, int32_t dim, mpm_dtype dtype, void* out_tokens,
+                                      int64_t* out_offsets, int32_t* out_map, void* stream);
+
+/*
  * Map composition across two insertions (Eq. 3): r*(p) = r2(r1(p)).
  *
  *   map1      int32 [rows0]: stage-1 map, local to image b of offsets0

@@ -27,7 +27,8 @@ STATUS_NAMES = {
     8: "MPM_ERR_ALIASING",
 }
 EXPORTS = ("mpm_abi_version", "mpm_status_string", "mpm_merge_workspace_size", "mpm_merge", "mpm_merge_timed",
-           "mpm_compose_maps", "mpm_unmerge_gather", "mpm_nearest_neighbors", "mpm_get_device_status")
+           "mpm_compose_maps", "mpm_unmerge_gather", "mpm_nearest_neighbors", "mpm_get_device_status",
+           "mpm_merge_no_alloc")
 
 _lib = None
 
@@ -53,6 +54,7 @@ def _declare(lib: ctypes.CDLL) -> None:
         "mpm_nearest_neighbors": (ctypes.c_int, [P, P, I32, I64, I32, ctypes.c_int, ctypes.c_int, P, P, P,
                                                  SZ, P]),
         "mpm_get_device_status": (ctypes.c_int, [P, P, P]),
+        "mpm_merge_no_alloc": (ctypes.c_int, [P, P, I32, I64, I32, ctypes.c_int, P, P, P, P]),
     }
     for name, (res, args) in sigs.items():
         fn = getattr(lib, name)
@@ -227,3 +229,26 @@ def device_status(workspace: torch.Tensor) -> int:
         _check("mpm_get_device_status",
                library().mpm_get_device_status(_ptr(workspace), ctypes.byref(code), _stream(dev)))
     return int(code.value)
+
+
+def merge_no_alloc(tokens: torch.Tensor, offsets: torch.Tensor, out_tokens: torch.Tensor,
+                   out_offsets: torch.Tensor, out_map: torch.Tensor):
+    """merge() for callers that cannot allocate device memory.
+
+    The caller provides every output buffer; the scratch space is a fixed
+    array inside the library (see mpm_merge_no_alloc in include/mpm.h for the
+    size limit, the first-call set-up and why overlapping calls race).
+    """
+    _cuda(tokens, "tokens", ndim=2)
+    _cuda(offsets, "offsets", torch.int64, 1)
+    _cuda(out_tokens, "out_tokens", tokens.dtype, 2)
+    _cuda(out_offsets, "out_offsets", torch.int64, 1)
+    _cuda(out_map, "out_map", torch.int32, 1)
+    dev = tokens.device
+    rows, dim = tokens.shape
+    with torch.cuda.device(dev):
+        code = library().mpm_merge_no_alloc(_ptr(tokens), _ptr(offsets), offsets.numel() - 1, rows, dim,
+                                            _dtype_code(tokens), _ptr(out_tokens), _ptr(out_offsets),
+                                            _ptr(out_map), _stream(dev))
+    _check("mpm_merge_no_alloc", code)
+    return out_tokens, out_offsets, out_map
