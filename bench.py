@@ -10,8 +10,8 @@ encoder blocks; it is not part of MPM and is not timed.
   python bench.py --impl reference ...   # the fp64 CPU oracle on host cores
 
 Timing: CUDA events on the launch stream bracket the two timed segments of
-every step (merge 1; merge 2 + compose + gather); L2 is flushed by a 256 MiB
-write before every step; W untimed warm-up steps; barrier + synchronize on
+every step (merge 1; merge 2 + compose + gather); L2 is flushed before every
+step by writing and then reading a 256 MiB buffer; W untimed warm-up steps; barrier + synchronize on
 both sides; the max over ranks is reported.  Each rank processes its own
 batch (images are independent: replicas, weak scaling, no collective on the
 data path).  One JSON line is printed by rank 0.
@@ -25,7 +25,6 @@ import json
 import os
 import platform
 import statistics
-import subprocess
 import sys
 import time
 
@@ -49,8 +48,8 @@ TRAFFIC_FILE = os.path.join(ROOT, "profiles", "affinity_tc_traffic.txt")
 def parse_args():
     p = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=20)
-    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--steps", type=int, default=200)
+    p.add_argument("--warmup", type=int, default=10)
     p.add_argument("--impl", choices=["mpm", "reference"], default="mpm")
     p.add_argument("--workload", default=DEFAULT_WORKLOAD)
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -85,7 +84,7 @@ def workload_desc(cfg, batch):
         "dim": int(cfg.dim),
         "insertions": int(cfg.insertions),
         "seed": int(cfg.seed),
-        "l2": "flushed by a 256 MiB write before every step",
+        "l2": "flushed before every step: 256 MiB written, then read back (clean lines)",
         "untimed": "the seeded N(0,0.05^2) stand-in for the encoder blocks between the two merges",
         "parallelism": "replicas (each rank merges its own batch; no data-path collective)",
     }
@@ -184,64 +183,108 @@ def run_reference(args):
 # Clock sampling during the timed region
 # ---------------------------------------------------------------------------
 class ClockSampler:
-    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
-             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
-             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    """SM clock and throttle reasons sampled during the timed region.
 
-    def __init__(self, gpu_index: int):
-        self.proc = None
-        self.gpu = gpu_index
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{gpu_index}.csv")
+    Reads NVML through ctypes (read-only queries: current and maximum SM
+    clock, clock event reasons) every millisecond from a thread, so that even
+    a timed region of a few milliseconds gets samples.  Falls back to
+    nothing (clocks null) when NVML is not available.
+    """
+
+    REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
+               0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown"}
+
+    def __init__(self, torch_device):
+        import ctypes
+        import threading
+
+        self.ok = False
+        self.samples = []
+        self.max_mhz = None
+        self._stop = threading.Event()
+        self._thread = None
+        try:
+            nvml = ctypes.CDLL("libnvidia-ml.so.1")
+            if nvml.nvmlInit_v2() != 0:
+                return
+            handle = ctypes.c_void_p()
+            bus = self._bus_id(torch_device)
+            if bus is None or nvml.nvmlDeviceGetHandleByPciBusId_v2(bus.encode(), ctypes.byref(handle)) != 0:
+                if nvml.nvmlDeviceGetHandleByIndex_v2(torch_device.index or 0, ctypes.byref(handle)) != 0:
+                    return
+            mx = ctypes.c_uint(0)
+            if nvml.nvmlDeviceGetMaxClockInfo(handle, 1, ctypes.byref(mx)) == 0:  # 1 = SM clock
+                self.max_mhz = float(mx.value)
+            self.reasons_fn = getattr(nvml, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+                getattr(nvml, "nvmlDeviceGetCurrentClocksThrottleReasons")
+            self.nvml, self.handle, self.ok = nvml, handle, True
+        except (OSError, AttributeError):
+            self.ok = False
+
+    @staticmethod
+    def _bus_id(dev):
+        import torch
+
+        props = torch.cuda.get_device_properties(dev)
+        try:
+            return f"{props.pci_domain_id:08X}:{props.pci_bus_id:02X}:{props.pci_device_id:02X}.0"
+        except AttributeError:
+            return None
+
+    def _run(self):
+        import ctypes
+
+        clk = ctypes.c_uint(0)
+        rsn = ctypes.c_ulonglong(0)
+        while not self._stop.is_set():
+            if self.nvml.nvmlDeviceGetClockInfo(self.handle, 1, ctypes.byref(clk)) == 0:
+                bits = rsn.value if self.reasons_fn(self.handle, ctypes.byref(rsn)) == 0 else 0
+                self.samples.append((float(clk.value), int(bits)))
+            time.sleep(0.001)
 
     def start(self):
-        try:
-            os.makedirs(os.path.dirname(self.path), exist_ok=True)
-            self.fh = open(self.path, "w")
-            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.QUERY}",
-                                          "--format=csv,noheader,nounits", "-lms", "100"],
-                                         stdout=self.fh, stderr=subprocess.DEVNULL)
-        except OSError:
-            self.proc = None
+        if not self.ok:
+            return
+        import threading
+
+        self._thread = threading.Thread(target=self._run, daemon=True)
+        self._thread.start()
+        t0 = time.perf_counter()
+        while not self.samples and time.perf_counter() - t0 < 1.0:
+            time.sleep(0.001)
 
     def stop(self):
-        if self.proc is None:
+        if not self.ok or self._thread is None:
             return None
-        self.proc.terminate()
-        try:
-            self.proc.wait(timeout=5)
-        except subprocess.TimeoutExpired:
-            self.proc.kill()
-        self.fh.close()
-        sm, smax, reasons = [], [], set()
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        with open(self.path) as f:
-            for line in f:
-                parts = [p.strip() for p in line.split(",")]
-                if len(parts) < 9:
-                    continue
-                try:
-                    sm.append(float(parts[1]))
-                    smax.append(float(parts[2]))
-                except ValueError:
-                    continue
-                for name, flag in zip(names, parts[5:9]):
-                    if flag.lower() == "active":
-                        reasons.add(name)
-        if not sm:
+        self._stop.set()
+        self._thread.join(timeout=5)
+        if not self.samples:
             return None
-        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
-                "samples": len(sm)}
+        reasons = set()
+        for _, bits in self.samples:
+            for bit, name in self.REASONS.items():
+                if bits & bit:
+                    reasons.add(name)
+        sm = [c for c, _ in self.samples]
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": self.max_mhz, "reasons": sorted(reasons),
+                "samples": len(sm), "source": "NVML, 1 ms period, during the timed steps"}
 
 
-def traffic_for(kernel_file: str):
-    """DRAM bytes per launch from the committed ncu summary, if the kernel is unchanged."""
+def traffic_for(kernel_file: str, rows_per_launch: float):
+    """DRAM bytes per launch from the committed ncu record, if the kernel is unchanged.
+
+    The record holds one captured launch's dram read + write bytes and its
+    rows; the kernel reads its input once, so the bytes scale with the rows.
+    """
     try:
         with open(TRAFFIC_FILE) as f:
             fields = dict(line.strip().split("=", 1) for line in f if "=" in line and not line.startswith("#"))
         with open(kernel_file, "rb") as f:
             sha = hashlib.sha256(f.read()).hexdigest()[:16]
         if fields.get("source_sha256_16") == sha:
-            return float(fields["dram_bytes_per_launch"])
+            per_row = (float(fields["dram_read_bytes"]) + float(fields["dram_write_bytes"])) / \
+                float(fields["rows_captured"])
+            return per_row * rows_per_launch
     except (OSError, ValueError, KeyError):
         pass
     return None
@@ -293,6 +336,7 @@ def run_mpm(args):
     rstar = torch.empty_like(m1)
     up = torch.empty_like(x0)
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    flush_sum = torch.zeros((), dtype=torch.int64, device=dev)
 
     # One untimed pass fixes the stage-1 counts, hence the stand-in noise.
     mpm.merge(x0, off0, workspace=ws, out_tokens=x1, out_offsets=off1, out_map=m1)
@@ -315,7 +359,10 @@ def run_mpm(args):
             self.cg = new_events(2)        # between compose and gather
 
     def step(ev: StepEvents, host_in=None, host_out=None):
+        # Evict the L2: write 256 MiB, then read it back so that the lines left
+        # behind are clean (no write-back lands on the first timed kernel).
         flush.fill_(1)
+        flush_sum.copy_(flush.view(torch.int64).sum())
         ev.seg[0].record(stream)
         if host_in is not None:
             x0.copy_(host_in[0], non_blocking=True)
@@ -357,7 +404,7 @@ def run_mpm(args):
     for _ in range(args.warmup):
         step(warm)
     assert mpm.device_status(ws) == 0, "device status reported an error during warm-up"
-    clocks = ClockSampler(local)
+    clocks = ClockSampler(dev)
     barrier()
     clocks.start()
     wall0 = time.perf_counter()
@@ -396,7 +443,8 @@ def run_mpm(args):
     achieved_tflops = sum(aff_flops) / (sum(aff_ms) * 1e-3) / 1e12
     flops_per_launch = sum(aff_flops) / launches
     tensor_peak = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
-    traffic = traffic_for(os.path.join(ROOT, "paper_2604_05718_gb300", "csrc", "affinity_tc.cu"))
+    rows_per_launch = (n0.sum() + (n1.sum() if two else 0.0)) / (2.0 if two else 1.0)
+    traffic = traffic_for(os.path.join(ROOT, "paper_2604_05718_gb300", "csrc", "affinity_tc.cu"), rows_per_launch)
     roofline = {
         "kernel": "affinity_tc (fused cosine affinity + arg max, tcgen05)",
         "bound": "tensor", "achieved": achieved_tflops, "peak": tensor_peak, "unit": "TFLOP/s",
