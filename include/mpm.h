@@ -73,9 +73,11 @@ typedef enum mpm_status {
 
 /* Which kernel computes the nearest neighbours (Eq. 1 + arg max). */
 typedef enum mpm_nn_algo {
-  MPM_NN_AUTO = 0,    /* tensor cores for bf16, CUDA-core fp32 otherwise */
-  MPM_NN_SIMT = 1,    /* CUDA-core fp32 FMA tiles (any dtype) */
-  MPM_NN_TCGEN05 = 2  /* TMA + tcgen05 MMA into TMEM (bf16 only) */
+  MPM_NN_AUTO = 0,        /* MPM_NN_TCGEN05_SYM for bf16, MPM_NN_SIMT for fp32 */
+  MPM_NN_SIMT = 1,        /* CUDA-core fp32 FMA tiles (any dtype) */
+  MPM_NN_TCGEN05 = 2,     /* TMA + tcgen05 MMA into TMEM, every tile of X X^T (bf16) */
+  MPM_NN_TCGEN05_SYM = 3  /* as above, tiles on or above the diagonal only, each
+                             feeding both its rows and its columns (bf16) */
 } mpm_nn_algo;
 
 /* Version of this ABI (MPM_ABI_VERSION). */

@@ -6,7 +6,7 @@
 // tensor-core precision would not be faithful to the fp32 definition.
 #include <math.h>
 
-#include "../../include/mpm.h"
+#include "mpm.h"
 #include "common.cuh"
 
 namespace mpm {
@@ -100,7 +100,7 @@ __global__ void __launch_bounds__(kThreads) affinity_simt_kernel(const uint8_t* 
 
 }  // namespace
 
-AffinityTile simt_tile() { return {BM, BN}; }
+AffinityTile simt_tile() { return {BM, BN, false}; }
 
 cudaError_t launch_affinity_simt(const void* tokens, int batch, int dim, bool bf16, const Workspace& ws,
                                  int num_sms, cudaStream_t stream) {

@@ -1,27 +1,39 @@
 // Tensor-core affinity + arg max for bf16 tokens (Eq. 1 and Algorithm 1
 // step 3), the one dense contraction of MPM.
 //
-// For every image b and every 128 x 256 tile of its N_b x N_b dot-product
-// matrix X X^T, the kernel
-//   * stages 128 rows (A) and 256 rows (B) of the RAW bf16 tokens, 64
-//     features at a time, into shared memory with TMA (128-byte swizzle);
-//   * accumulates A B^T in fp32 in tensor memory with tcgen05.mma
-//     (M = 128, N = 256, K = 16 per instruction; bf16 products are exact in
-//     fp32);
-//   * reads the accumulator back with tcgen05.ld and scales column j by
-//     1/max(|x_j|, 1e-12) in fp32.  Because 1/|x_i| is constant along a row,
-//     the row arg max of this score is the arg max of the cosine S_ij.  The
-//     diagonal and columns outside the image are skipped; a running
-//     (max, lowest j) per row is merged into the packed 64-bit key with
+// For an image b, G = X X^T holds the dot products of its raw bf16 tokens.
+// The kernel
+//   * stages 128 rows (A) and 256 rows (B) of the RAW tokens, 64 features at
+//     a time, into shared memory with TMA (128-byte swizzle);
+//   * accumulates a 128 x 256 tile of G in fp32 in tensor memory with
+//     tcgen05.mma (M = 128, N = 256, K = 16 per instruction; bf16 products
+//     are exact in fp32);
+//   * reads the tile back with tcgen05.ld and turns it into arg-max
+//     candidates: row i scores column j by G_ij / max(|x_j|, 1e-12) in fp32
+//     (the row factor 1/|x_i| of the cosine does not change a row's arg
+//     max).  The diagonal and columns outside the image are skipped, and a
+//     running (max, lowest j) per row goes into a packed 64-bit key with
 //     atomicMax.  The N x N matrix never reaches global memory.
+//
+// Dense mode computes every tile of G.  Symmetric mode (the default) uses
+// G_ij = G_ji.  With 128-wide blocks I (rows) and J (columns), it computes
+// only the tiles that contain a block with J >= I.  From an off-diagonal
+// block it takes both the row candidates (rows of I over columns of J) and
+// the column candidates: row j of block J scores row i of block I by
+// G_ij / |x_i|, which is the same quantity its own row would have produced.
+// A warp max and a ballot per column of each 32 x 32 block give every
+// column its best (score, lowest i).  Shared-memory 64-bit atomicMax combines the four row
+// groups, and the last warp to finish a tile flushes the 256 column keys to
+// global memory.  Both modes merge candidates with the same packed-key
+// atomicMax, so the result does not depend on which tile saw a pair first.
 //
 // The kernel is persistent (one CTA per SM) and warp-specialised:
 //   warp 0    TMA producer (4-stage shared-memory ring)
 //   warp 1    TMEM allocator and MMA issuer (two 256-column accumulators)
-//   warps 2-9 epilogue: each of the 4 TMEM lane groups is read by two warps,
-//             one per 128-column half, so a tile's epilogue overlaps the
-//             next tile's MMAs.
-// Every wait is bounded; on expiry the kernel records
+//   warps 2-17 epilogue: each of the 4 TMEM lane groups (32 rows) is read by
+//             four warps, one per 64-column quarter, so a tile's epilogue
+//             overlaps the next tile's MMAs.
+// Every wait is bounded.  On expiry the kernel records
 // MPM_ERR_DEVICE_TIMEOUT, lets in-flight copies and MMAs finish, frees its
 // tensor memory and returns.
 #include <cuda.h>
@@ -31,22 +43,23 @@
 #include <atomic>
 #include <mutex>
 
-#include "../../include/mpm.h"
+#include "mpm.h"
 #include "common.cuh"
 #include "ptx.cuh"
 
 namespace mpm {
 namespace {
 
-constexpr int BM = 128;                        // tile rows = TMEM lanes
-constexpr int BN = 256;                        // tile columns = MMA N
+constexpr int BM = 128;                        // tile rows = TMEM lanes = one 128 block
+constexpr int BN = 256;                        // tile columns = MMA N = two 128 blocks
 constexpr int BK = 64;                         // bf16 features per swizzled row
 constexpr int TMA_ROWS = 128;                  // rows per TMA box
 constexpr int STAGES = 4;
 constexpr int A_BYTES = BM * BK * 2;           // 16 KiB
 constexpr int B_BYTES = BN * BK * 2;           // 32 KiB
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-constexpr int EPI_WARPS = 8;
+constexpr int EPI_WARPS = 16;                  // 4 per TMEM lane group, 64 columns each
+constexpr int EPI_COLS = BN / (EPI_WARPS / 4);  // columns read by one epilogue warp
 constexpr int THREADS = (2 + EPI_WARPS) * 32;
 constexpr uint32_t TMEM_COLS = 2 * BN;         // double-buffered accumulator
 constexpr uint32_t IDESC = ptx::idesc_bf16_f32(BM, BN);
@@ -59,6 +72,8 @@ struct Control {
   uint64_t acc_empty[2];       // epilogue finished reading accumulator a
   uint64_t scale_ready[2];     // column scales of accumulator a written
   uint64_t drain;              // all MMAs completed (teardown)
+  unsigned long long colkey[2][BN];  // symmetric mode: column candidates of accumulator a
+  int colcount[2];             // epilogue warps done with accumulator a's column keys
   uint32_t tmem_base;
   int abort_flag;
 };
@@ -69,19 +84,38 @@ constexpr size_t SMEM_BYTES = 1024 + static_cast<size_t>(STAGES) * STAGE_BYTES +
 struct Item {
   int64_t base;  // first row of the image
   int n;         // tokens in the image
-  int row0;      // first local row of the tile
-  int col0;      // first local column of the tile
+  int row0;      // first local row of the tile (row block I = row0 / 128)
+  int col0;      // first local column of the tile (column blocks 2T, 2T+1 with T = col0 / 256)
 };
 
+template <bool SYM>
 __device__ __forceinline__ Item decode_item(const Workspace& ws, int batch, int64_t w) {
   const int b = find_item_image(ws.plan, batch, w);
-  const int64_t local = w - __ldg(ws.plan + b);
+  int64_t local = w - __ldg(ws.plan + b);
   Item it;
   it.base = __ldg(ws.soff + b);
   it.n = static_cast<int>(__ldg(ws.soff + b + 1) - it.base);
-  const int ct = (it.n + BN - 1) / BN;
-  it.row0 = static_cast<int>(local / ct) * BM;
-  it.col0 = static_cast<int>(local % ct) * BN;
+  const int64_t c = (it.n + BN - 1) / BN;
+  if (!SYM) {
+    it.row0 = static_cast<int>(local / c) * BM;
+    it.col0 = static_cast<int>(local % c) * BN;
+    return it;
+  }
+  // Symmetric tiling (see affinity_tiles): row blocks 2m and 2m+1 start at
+  // prefix P(m) = 2mC - m(m-1); find the last pair whose prefix is <= local
+  // by bisection, then the block within the pair.
+  const int64_t r = (it.n + BM - 1) / BM;
+  int64_t lo = 0, hi = (r - 1) / 2;
+  while (lo < hi) {
+    const int64_t mid = (lo + hi + 1) / 2;
+    if (2 * mid * c - mid * (mid - 1) <= local) lo = mid; else hi = mid - 1;
+  }
+  local -= 2 * lo * c - lo * (lo - 1);
+  const int64_t per = c - lo;  // tiles of each row block of the pair
+  const int64_t blk = 2 * lo + (local >= per ? 1 : 0);
+  if (local >= per) local -= per;
+  it.row0 = static_cast<int>(blk) * BM;
+  it.col0 = static_cast<int>(lo + local) * BN;
   return it;
 }
 
@@ -90,6 +124,65 @@ __device__ __forceinline__ void fail(Control* ctl, int32_t* status, int32_t role
   report(status, MPM_ERR_DEVICE_TIMEOUT, role);
 }
 
+// Signed-integer order of fp32 values: a < b as floats iff f(a) < f(b) as
+// int32 (negative floats have their magnitude bits flipped).  f(x) with the
+// sign bit flipped equals order_f32(x).  -0 sorts below +0, so scores are
+// canonicalised first.
+__device__ __forceinline__ int float_order_s32(float x) {
+  const int b = __float_as_int(x);
+  return b ^ ((b >> 31) & 0x7FFFFFFF);
+}
+
+// One 32-column chunk of the epilogue for the thread's row: row candidates
+// (best column by G_ij / |x_j|), skipping the diagonal when DIAG, and, when
+// COL, the column candidates (best row of the warp by G_ij / |x_i|).
+template <bool DIAG, bool COL>
+__device__ __forceinline__ void epilogue_chunk(const uint32_t (&v)[32], const float* sc, int c, int jd,
+                                               float& best, int& bj, float inv_i, int lane, int row_base,
+                                               int n, int col0, unsigned long long* colkey) {
+#pragma unroll
+  for (int k = 0; k < 32; k += 4) {
+    const float4 s4 = *reinterpret_cast<const float4*>(sc + c + k);
+    const float sv[4] = {s4.x, s4.y, s4.z, s4.w};
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const float s = __uint_as_float(v[k + u]) * sv[u];
+      if (s > best && (!DIAG || c + k + u != jd)) {
+        best = s;
+        bj = c + k + u;
+      }
+    }
+  }
+  if (COL) {
+    // Column j = col0 + c + k scores this row by G_ij / |x_i|.  fma(v, inv, +0)
+    // is the rounded product with -0 folded into +0, so equal scores order
+    // equally.  Per column: the warp's best ordered score (one warp max) and
+    // the lanes holding it (one ballot); lane k keeps column k's result.
+    // Rows outside the image only occur in an image's last row block, whose
+    // column updates (blocks J > I) lie wholly outside the image and are
+    // dropped by the column check; the row check below is a second guard.
+    int top = 0;
+    uint32_t lanes = 0;
+#pragma unroll
+    for (int k = 0; k < 32; ++k) {
+      const int key = float_order_s32(__fmaf_rn(__uint_as_float(v[k]), inv_i, 0.0f));
+      const int m = __reduce_max_sync(0xFFFFFFFFu, key);
+      const uint32_t ball = __ballot_sync(0xFFFFFFFFu, key == m);
+      if (lane == k) {
+        top = m;
+        lanes = ball;
+      }
+    }
+    const int winner = row_base + __ffs(static_cast<int>(lanes)) - 1;
+    if (winner < n && col0 + c + lane < n) {
+      const uint32_t hi = static_cast<uint32_t>(top) ^ 0x80000000u;  // = order_f32 of the score
+      atomicMax(colkey + c + lane, (static_cast<unsigned long long>(hi) << 32) |
+                                       static_cast<unsigned long long>(0xFFFFFFFFu - static_cast<uint32_t>(winner)));
+    }
+  }
+}
+
+template <bool SYM>
 __global__ void __launch_bounds__(THREADS, 1)
     affinity_tc_kernel(const __grid_constant__ CUtensorMap tmap, int batch, int ksteps, Workspace ws) {
   extern __shared__ uint8_t smem_raw[];
@@ -108,11 +201,15 @@ __global__ void __launch_bounds__(THREADS, 1)
       ptx::mbar_init(&ctl->acc_full[a], 1);
       ptx::mbar_init(&ctl->acc_empty[a], EPI_WARPS * 32);
       ptx::mbar_init(&ctl->scale_ready[a], EPI_WARPS * 32);
+      ctl->colcount[a] = 0;
     }
     ptx::mbar_init(&ctl->drain, 1);
     ctl->abort_flag = 0;
     ptx::fence_barrier_init();
     ptx::prefetch_tensor_map(&tmap);
+  }
+  if (SYM) {
+    for (int e = threadIdx.x; e < 2 * BN; e += THREADS) (&ctl->colkey[0][0])[e] = 0ull;
   }
   if (warp == 1) {
     ptx::tmem_alloc(&ctl->tmem_base, TMEM_COLS);
@@ -134,7 +231,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       uint32_t issued_phase = 0;      // bit s: parity of that load's phase
       bool ok = true;
       for (int64_t w = blockIdx.x; ok && w < total; w += gridDim.x) {
-        const Item it = decode_item(ws, batch, w);
+        const Item it = decode_item<SYM>(ws, batch, w);
         const int32_t arow = static_cast<int32_t>(it.base + it.row0);
         const int32_t brow = static_cast<int32_t>(it.base + it.col0);
         for (int kb = 0; kb < ksteps; ++kb) {
@@ -213,17 +310,17 @@ __global__ void __launch_bounds__(THREADS, 1)
     __syncwarp();
   } else {
     // ---------------- epilogue ----------------
-    const int ew = warp - 2;                 // 0..7
+    const int ew = warp - 2;                 // 0..EPI_WARPS-1
     const int q = warp & 3;                  // TMEM lane group of this warp
-    const int half = ew >> 2;                // 128-column half of the tile
-    const int et = ew * 32 + lane;           // 0..255: column whose scale this thread loads
+    const int quarter = ew >> 2;             // 64-column slice of the tile
+    const int et = ew * 32 + lane;           // column whose scale this thread loads (if < BN)
     const uint32_t lane_addr = static_cast<uint32_t>(q * 32) << 16;
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int64_t w = blockIdx.x; w < total; w += gridDim.x) {
-      const Item it = decode_item(ws, batch, w);
+      const Item it = decode_item<SYM>(ws, batch, w);
       float* sc = scale + acc * BN;
-      {
+      if (et < BN) {
         const int j = it.col0 + et;
         sc[et] = j < it.n ? __ldg(ws.inv_norm + it.base + j) : __int_as_float(0x7fc00000);  // NaN never wins
       }
@@ -234,32 +331,59 @@ __global__ void __launch_bounds__(THREADS, 1)
         break;
       }
       ptx::tc_fence_after_sync();
-      const int row = it.row0 + q * 32 + lane;     // local row owned by this thread
+      const int row_base = it.row0 + q * 32;
+      const int row = row_base + lane;             // local row owned by this thread
       const int jd = row - it.col0;                // its diagonal column within the tile
+      const int c0 = quarter * EPI_COLS;           // first tile column of this warp
+      const int iblk = it.row0 / BM;
+      const int jblk = (it.col0 + c0) / BM;        // the 128-column block of this warp's slice
+      // Symmetric mode skips blocks below the diagonal (their pairs come from
+      // the mirrored block) and takes column candidates above it.
+      const bool diag = jblk == iblk;
+      const bool read = !SYM || jblk >= iblk;
+      const bool col_update = SYM && jblk > iblk;
+      const float inv_i = (col_update && row < it.n) ? __ldg(ws.inv_norm + it.base + row) : 0.f;
       float best = -INFINITY;
       int bj = -1;
+      if (read) {
 #pragma unroll 1
-      for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 32) {
-        uint32_t v[32];
-        ptx::tmem_ld_32x32b_x32(tmem + lane_addr + static_cast<uint32_t>(acc * BN + c), v);
-        ptx::tmem_wait_ld(v);
-#pragma unroll
-        for (int k = 0; k < 32; k += 4) {
-          const float4 s4 = *reinterpret_cast<const float4*>(sc + c + k);
-          const float sv[4] = {s4.x, s4.y, s4.z, s4.w};
-#pragma unroll
-          for (int u = 0; u < 4; ++u) {
-            const float s = __uint_as_float(v[k + u]) * sv[u];
-            if (s > best && c + k + u != jd) {
-              best = s;
-              bj = c + k + u;
-            }
+        for (int c = c0; c < c0 + EPI_COLS; c += 32) {
+          uint32_t v[32];
+          ptx::tmem_ld_32x32b_x32(tmem + lane_addr + static_cast<uint32_t>(acc * BN + c), v);
+          ptx::tmem_wait_ld(v);
+          unsigned long long* ck = ctl->colkey[acc];
+          if (diag) {
+            epilogue_chunk<true, false>(v, sc, c, jd, best, bj, inv_i, lane, row_base, it.n, it.col0, ck);
+          } else if (col_update) {
+            epilogue_chunk<false, true>(v, sc, c, jd, best, bj, inv_i, lane, row_base, it.n, it.col0, ck);
+          } else {
+            epilogue_chunk<false, false>(v, sc, c, jd, best, bj, inv_i, lane, row_base, it.n, it.col0, ck);
           }
         }
       }
       ptx::tc_fence_before_sync();
       ptx::mbar_arrive(&ctl->acc_empty[acc]);
       if (bj >= 0 && row < it.n) atomicMax(ws.keys + it.base + row, make_key(best, it.col0 + bj));
+      if (SYM) {
+        // The last epilogue warp to finish this tile flushes its column keys.
+        __threadfence_block();
+        __syncwarp();
+        int last = 0;
+        if (lane == 0) last = atomicAdd(&ctl->colcount[acc], 1) == EPI_WARPS - 1;
+        last = __shfl_sync(0xFFFFFFFFu, last, 0);
+        if (last) {
+          __threadfence_block();
+          for (int e = lane; e < BN; e += 32) {
+            const unsigned long long k = ctl->colkey[acc][e];
+            if (k != 0ull) {
+              atomicMax(ws.keys + it.base + it.col0 + e, k);
+              ctl->colkey[acc][e] = 0ull;
+            }
+          }
+          if (lane == 0) ctl->colcount[acc] = 0;
+          __threadfence_block();
+        }
+      }
       if (++acc == 2) {
         acc = 0;
         acc_phase ^= 1u;
@@ -289,14 +413,32 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
   return fn;
 }
 
+// The shared-memory opt-in is a per-device attribute: set it once per
+// device and kernel instance.
+template <bool SYM>
+cudaError_t ensure_smem_attr() {
+  static std::atomic<uint64_t> done{0};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const uint64_t bit = 1ull << (dev & 63);
+  if (!(done.load() & bit)) {
+    e = cudaFuncSetAttribute(affinity_tc_kernel<SYM>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(SMEM_BYTES));
+    if (e != cudaSuccess) return e;
+    done.fetch_or(bit);
+  }
+  return cudaSuccess;
+}
+
 }  // namespace
 
-AffinityTile tc_tile() { return {BM, BN}; }
+AffinityTile tc_tile(bool symmetric) { return {BM, BN, symmetric}; }
 
 bool tc_available() { return get_encode() != nullptr; }
 
-cudaError_t launch_affinity_tc(const void* tokens, int batch, int64_t rows, int dim, const Workspace& ws,
-                               int num_sms, cudaStream_t stream) {
+cudaError_t launch_affinity_tc(const void* tokens, int batch, int64_t rows, int dim, bool symmetric,
+                               const Workspace& ws, int num_sms, cudaStream_t stream) {
   PFN_cuTensorMapEncodeTiled_v12000 encode = get_encode();
   if (encode == nullptr) return cudaErrorNotSupported;
   CUtensorMap map;
@@ -308,20 +450,18 @@ cudaError_t launch_affinity_tc(const void* tokens, int batch, int64_t rows, int 
              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return cudaErrorInvalidValue;
-  // The shared-memory opt-in is a per-device attribute: set it once per device.
-  static std::atomic<uint64_t> attr_done{0};
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return e;
-  const uint64_t bit = 1ull << (dev & 63);
-  if (!(attr_done.load() & bit)) {
-    e = cudaFuncSetAttribute(affinity_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(SMEM_BYTES));
-    if (e != cudaSuccess) return e;
-    attr_done.fetch_or(bit);
-  }
   const int ksteps = (dim + BK - 1) / BK;
-  affinity_tc_kernel<<<num_sms > 0 ? num_sms : 1, THREADS, SMEM_BYTES, stream>>>(map, batch, ksteps, ws);
+  const int grid = num_sms > 0 ? num_sms : 1;
+  cudaError_t e;
+  if (symmetric) {
+    e = ensure_smem_attr<true>();
+    if (e != cudaSuccess) return e;
+    affinity_tc_kernel<true><<<grid, THREADS, SMEM_BYTES, stream>>>(map, batch, ksteps, ws);
+  } else {
+    e = ensure_smem_attr<false>();
+    if (e != cudaSuccess) return e;
+    affinity_tc_kernel<false><<<grid, THREADS, SMEM_BYTES, stream>>>(map, batch, ksteps, ws);
+  }
   return cudaGetLastError();
 }
 

@@ -36,6 +36,17 @@ __device__ __forceinline__ int find_item_image(const int64_t* __restrict__ plan,
   return lo;
 }
 
+// Work items (tiles) of the affinity pass for one image of n tokens.  Dense:
+// every rows x cols tile.  Symmetric (cols == 2 * rows): row block I needs
+// only the column tiles T holding a block J >= I, i.e. 2T + 1 >= I, so it
+// has C - (I >> 1) of them; row blocks 2m and 2m+1 have 2(C - m) together.
+__host__ __device__ __forceinline__ int64_t affinity_tiles(int64_t n, int rows, int cols, bool symmetric) {
+  const int64_t r = (n + rows - 1) / rows, c = (n + cols - 1) / cols;
+  if (!symmetric) return r * c;
+  const int64_t q = r / 2;
+  return 2 * q * c - q * (q - 1) + (r & 1) * (c - q);
+}
+
 // A total order on floats as unsigned integers (larger float -> larger key).
 __device__ __forceinline__ uint32_t order_f32(float f) {
   uint32_t u = __float_as_uint(f);

@@ -5,13 +5,15 @@
 // warp per row; grids are sized from the SM count and loop over rows.
 #include <math.h>
 
-#include "../../include/mpm.h"
+#include "mpm.h"
 #include "common.cuh"
 
 namespace mpm {
 namespace {
 
 constexpr int kThreads = 256;
+constexpr int kPrepRows = 2;   // rows per warp iteration in prep_kernel
+constexpr int kPrepVecs = 4;   // 16-byte vectors per lane and row per pass
 
 __device__ __forceinline__ int64_t clamp64(int64_t v, int64_t lo, int64_t hi) {
   return v < lo ? lo : (v > hi ? hi : v);
@@ -37,7 +39,7 @@ struct ImageCursor {
 __global__ void __launch_bounds__(kThreads) prep_kernel(const uint8_t* __restrict__ tokens,
                                                         const int64_t* __restrict__ offsets,
                                                         int batch, int64_t rows, int row_bytes,
-                                                        bool bf16, int tile_m, int tile_n,
+                                                        bool bf16, AffinityTile tile,
                                                         Workspace ws) {
   if (blockIdx.x == 0) {
     __shared__ int64_t sh[32];
@@ -69,7 +71,7 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(const uint8_t* __restric
     }
     __syncthreads();
     if (threadIdx.x == 0 && bad >= 0) report(ws.status, MPM_ERR_DEVICE_CHECK, bad);
-    // plan[b] = sum_{b' < b} ceil(N_b'/tile_m) * ceil(N_b'/tile_n).
+    // plan[b] = number of affinity tiles of the images before b.
     __threadfence_block();
     int64_t acc = 0;
     for (int base = 0; base <= batch; base += kThreads) {
@@ -77,7 +79,7 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(const uint8_t* __restric
       int64_t items = 0;
       if (idx < batch) {
         const int64_t n = ws.soff[idx + 1] - ws.soff[idx];
-        items = ((n + tile_m - 1) / tile_m) * ((n + tile_n - 1) / tile_n);
+        items = affinity_tiles(n, tile.rows, tile.cols, tile.symmetric);
       }
       int64_t total;
       const int64_t incl = block_incl_sum<int64_t>(items, sh, &total);
@@ -87,20 +89,44 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(const uint8_t* __restric
   }
 
   // Inverse norms of every used row, and the arg-max keys reset to "none".
+  // Each warp takes kPrepRows consecutive rows at a time and issues all of
+  // their 16-byte loads before reducing, to keep enough bytes in flight.
   const int64_t used = clamp64(offsets[batch], 0, rows);
   const int lane = threadIdx.x & 31;
   const int64_t warp = (static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x) >> 5;
   const int64_t nwarps = (static_cast<int64_t>(gridDim.x) * kThreads) >> 5;
   const int nvec = row_bytes >> 4;
-  for (int64_t g = warp; g < used; g += nwarps) {
-    const uint4* src = reinterpret_cast<const uint4*>(tokens + g * row_bytes);
-    float s = 0.f;
-    for (int v = lane; v < nvec; v += 32) s += sumsq16(__ldg(src + v), bf16);
+  for (int64_t g0 = warp * kPrepRows; g0 < used; g0 += nwarps * kPrepRows) {
+    float s[kPrepRows];
 #pragma unroll
-    for (int d = 16; d > 0; d >>= 1) s += __shfl_xor_sync(0xFFFFFFFFu, s, d);
-    if (lane == 0) {
-      ws.inv_norm[g] = 1.0f / fmaxf(sqrtf(s), 1e-12f);
-      ws.keys[g] = 0ull;
+    for (int r = 0; r < kPrepRows; ++r) s[r] = 0.f;
+    for (int v0 = lane; v0 < nvec; v0 += 32 * kPrepVecs) {
+      uint4 buf[kPrepRows][kPrepVecs];
+#pragma unroll
+      for (int r = 0; r < kPrepRows; ++r) {
+        const uint4* src = reinterpret_cast<const uint4*>(tokens + (g0 + r) * row_bytes);
+#pragma unroll
+        for (int u = 0; u < kPrepVecs; ++u) {
+          const int v = v0 + 32 * u;
+          buf[r][u] = (g0 + r < used && v < nvec) ? __ldg(src + v) : make_uint4(0, 0, 0, 0);
+        }
+      }
+#pragma unroll
+      for (int r = 0; r < kPrepRows; ++r)
+#pragma unroll
+        for (int u = 0; u < kPrepVecs; ++u) s[r] += sumsq16(buf[r][u], bf16);
+    }
+#pragma unroll
+    for (int r = 0; r < kPrepRows; ++r) {
+#pragma unroll
+      for (int d = 16; d > 0; d >>= 1) s[r] += __shfl_xor_sync(0xFFFFFFFFu, s[r], d);
+    }
+    if (lane < kPrepRows && g0 + lane < used) {
+      float mine = s[0];
+#pragma unroll
+      for (int r = 1; r < kPrepRows; ++r) mine = lane == r ? s[r] : mine;
+      ws.inv_norm[g0 + lane] = 1.0f / fmaxf(sqrtf(mine), 1e-12f);
+      ws.keys[g0 + lane] = 0ull;
     }
   }
 }
@@ -168,7 +194,7 @@ __global__ void __launch_bounds__(kScanThreads) mutual_compact_kernel(int batch,
 // ---------------------------------------------------------------------------
 // Pair average + compaction (Eq. 2): one warp per output row.
 // ---------------------------------------------------------------------------
-template <int U>
+template <int R, int U>
 __global__ void __launch_bounds__(kThreads) pair_average_kernel(const uint8_t* __restrict__ tokens,
                                                                 uint8_t* __restrict__ out,
                                                                 int batch, int64_t rows, int row_bytes,
@@ -180,28 +206,48 @@ __global__ void __launch_bounds__(kThreads) pair_average_kernel(const uint8_t* _
   const int64_t total = clamp64(out_offsets[batch], 0, rows);
   const int nvec = row_bytes >> 4;
   ImageCursor cur;
-  for (int64_t t = warp; t < total; t += nwarps) {
-    cur.locate(out_offsets, batch, t);
-    const int64_t in_base = ws.soff[cur.b];
-    const int2 rep = ws.reps[in_base + (t - cur.lo)];
-    const uint4* a = reinterpret_cast<const uint4*>(tokens + (in_base + rep.x) * row_bytes);
-    const uint4* p = reinterpret_cast<const uint4*>(tokens + (in_base + (rep.y >= 0 ? rep.y : rep.x)) * row_bytes);
-    uint4* dst = reinterpret_cast<uint4*>(out + t * row_bytes);
+  // Each warp writes R consecutive output rows per iteration; all loads of
+  // a pass are issued before any store.
+  for (int64_t t0 = warp * R; t0 < total; t0 += nwarps * R) {
+    const uint4* a[R];
+    const uint4* p[R];
+    uint4* dst[R];
+    bool live[R], pair[R];
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      const int64_t t = t0 + r;
+      live[r] = t < total;
+      pair[r] = false;
+      a[r] = p[r] = nullptr;
+      dst[r] = reinterpret_cast<uint4*>(out + t * row_bytes);
+      if (live[r]) {
+        cur.locate(out_offsets, batch, t);
+        const int64_t in_base = ws.soff[cur.b];
+        const int2 rep = ws.reps[in_base + (t - cur.lo)];
+        pair[r] = rep.y >= 0;
+        a[r] = reinterpret_cast<const uint4*>(tokens + (in_base + rep.x) * row_bytes);
+        p[r] = reinterpret_cast<const uint4*>(tokens + (in_base + (pair[r] ? rep.y : rep.x)) * row_bytes);
+      }
+    }
     for (int v0 = lane; v0 < nvec; v0 += 32 * U) {
-      uint4 va[U], vb[U];
+      uint4 va[R][U], vb[R][U];
 #pragma unroll
-      for (int u = 0; u < U; ++u) {
-        const int v = v0 + 32 * u;
-        if (v < nvec) {
-          va[u] = __ldcs(a + v);
-          vb[u] = rep.y >= 0 ? __ldcs(p + v) : va[u];
+      for (int r = 0; r < R; ++r)
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+          const int v = v0 + 32 * u;
+          if (live[r] && v < nvec) {
+            va[r][u] = __ldcs(a[r] + v);
+            if (pair[r]) vb[r][u] = __ldcs(p[r] + v);
+          }
         }
-      }
 #pragma unroll
-      for (int u = 0; u < U; ++u) {
-        const int v = v0 + 32 * u;
-        if (v < nvec) dst[v] = rep.y >= 0 ? avg16(va[u], vb[u], bf16) : va[u];
-      }
+      for (int r = 0; r < R; ++r)
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+          const int v = v0 + 32 * u;
+          if (live[r] && v < nvec) dst[r][v] = pair[r] ? avg16(va[r][u], vb[r][u], bf16) : va[r][u];
+        }
     }
   }
 }
@@ -297,8 +343,7 @@ cudaError_t launch_prep(const void* tokens, const int64_t* offsets, int batch, i
                         cudaStream_t stream) {
   const int row_bytes = dim * (bf16 ? 2 : 4);
   prep_kernel<<<grid_for(num_sms, 8), kThreads, 0, stream>>>(
-      static_cast<const uint8_t*>(tokens), offsets, batch, rows, row_bytes, bf16, tile.rows,
-      tile.cols, ws);
+      static_cast<const uint8_t*>(tokens), offsets, batch, rows, row_bytes, bf16, tile, ws);
   return cudaGetLastError();
 }
 
@@ -312,7 +357,7 @@ cudaError_t launch_pair_average(const void* tokens, void* out_tokens, int batch,
                                 int dim, bool bf16, const Workspace& ws,
                                 const int64_t* out_offsets, int num_sms, cudaStream_t stream) {
   const int row_bytes = dim * (bf16 ? 2 : 4);
-  pair_average_kernel<4><<<grid_for(num_sms, 8), kThreads, 0, stream>>>(
+  pair_average_kernel<1, 4><<<grid_for(num_sms, 8), kThreads, 0, stream>>>(
       static_cast<const uint8_t*>(tokens), static_cast<uint8_t*>(out_tokens), batch, rows,
       row_bytes, bf16, ws, out_offsets);
   return cudaGetLastError();

@@ -23,9 +23,12 @@ struct Workspace {
 };
 
 // Tile of one affinity work item: rows x columns of the cosine matrix.
+// symmetric: only tiles holding a 128-block at or above the diagonal are
+// computed (requires cols == 2 * rows).
 struct AffinityTile {
   int rows;
   int cols;
+  bool symmetric;
 };
 
 // Inverse row norms, key reset, offsets sanitisation and the work plan.
@@ -38,10 +41,10 @@ cudaError_t launch_affinity_simt(const void* tokens, int batch, int dim, bool bf
                                  const Workspace& ws, int num_sms, cudaStream_t stream);
 AffinityTile simt_tile();
 
-// TMA + tcgen05 affinity + arg max (bf16).
-cudaError_t launch_affinity_tc(const void* tokens, int batch, int64_t rows, int dim,
+// TMA + tcgen05 affinity + arg max (bf16), dense or symmetric tiling.
+cudaError_t launch_affinity_tc(const void* tokens, int batch, int64_t rows, int dim, bool symmetric,
                                const Workspace& ws, int num_sms, cudaStream_t stream);
-AffinityTile tc_tile();
+AffinityTile tc_tile(bool symmetric);
 bool tc_available();
 
 // Mutual check, representative scan, per-image counts, output offsets.

@@ -6,7 +6,7 @@
 
 #include <atomic>
 
-#include "../../include/mpm.h"
+#include "mpm.h"
 #include "launch.h"
 
 namespace {
@@ -95,22 +95,28 @@ mpm_status check_tokens(const void* tokens, int64_t rows, int32_t dim, mpm_dtype
   return MPM_OK;
 }
 
+// Kernel used when the caller does not choose one: the symmetric tensor-core
+// kernel for bf16, CUDA-core fp32 FMA for fp32 (faithful to fp32 inputs).
+mpm_nn_algo default_algo(mpm_dtype dtype) { return dtype == MPM_BF16 ? MPM_NN_TCGEN05_SYM : MPM_NN_SIMT; }
+
 // The affinity + arg max stage shared by mpm_merge and mpm_nearest_neighbors.
 mpm_status run_affinity(const void* tokens, const int64_t* offsets, int32_t batch, int64_t rows, int32_t dim,
                         mpm_dtype dtype, mpm_nn_algo algo, const Workspace& ws, cudaStream_t stream) {
   const bool bf16 = dtype == MPM_BF16;
-  if (algo == MPM_NN_AUTO) algo = bf16 ? MPM_NN_TCGEN05 : MPM_NN_SIMT;
-  if (algo == MPM_NN_TCGEN05 && !bf16) return MPM_ERR_UNSUPPORTED;
-  if (algo != MPM_NN_SIMT && algo != MPM_NN_TCGEN05) return MPM_ERR_INVALID_ARG;
-  if (algo == MPM_NN_TCGEN05 && !mpm::tc_available()) return MPM_ERR_UNSUPPORTED;
+  if (algo == MPM_NN_AUTO) algo = default_algo(dtype);
+  const bool tc = algo == MPM_NN_TCGEN05 || algo == MPM_NN_TCGEN05_SYM;
+  if (algo != MPM_NN_SIMT && !tc) return MPM_ERR_INVALID_ARG;
+  if (tc && !bf16) return MPM_ERR_UNSUPPORTED;
+  if (tc && !mpm::tc_available()) return MPM_ERR_UNSUPPORTED;
   const int sms = num_sms();
   if (sms <= 0) return MPM_ERR_CUDA;
-  const mpm::AffinityTile tile = algo == MPM_NN_TCGEN05 ? mpm::tc_tile() : mpm::simt_tile();
+  const bool sym = algo == MPM_NN_TCGEN05_SYM;
+  const mpm::AffinityTile tile = tc ? mpm::tc_tile(sym) : mpm::simt_tile();
   cudaError_t e = mpm::launch_prep(tokens, offsets, batch, rows, dim, bf16, tile, ws, sms, stream);
   if (e != cudaSuccess) return MPM_ERR_CUDA;
   if (rows == 0) return MPM_OK;  // every image is empty: nothing to compare
-  if (algo == MPM_NN_TCGEN05) {
-    e = mpm::launch_affinity_tc(tokens, batch, rows, dim, ws, sms, stream);
+  if (tc) {
+    e = mpm::launch_affinity_tc(tokens, batch, rows, dim, sym, ws, sms, stream);
   } else {
     e = mpm::launch_affinity_simt(tokens, batch, dim, bf16, ws, sms, stream);
   }
@@ -176,8 +182,9 @@ mpm_status mpm_merge_timed(const void* tokens, const int64_t* offsets, int32_t b
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const Workspace ws = carve(workspace, rows, batch);
   const bool bf16 = dtype == MPM_BF16;
-  const mpm_nn_algo algo = bf16 ? MPM_NN_TCGEN05 : MPM_NN_SIMT;
-  if (algo == MPM_NN_TCGEN05 && !mpm::tc_available()) return MPM_ERR_UNSUPPORTED;
+  const mpm_nn_algo algo = default_algo(dtype);
+  const bool tc = algo != MPM_NN_SIMT;
+  if (tc && !mpm::tc_available()) return MPM_ERR_UNSUPPORTED;
   const int sms = num_sms();
   if (sms <= 0) return MPM_ERR_CUDA;
   // Records stage_events[idx] (if profiling) on the launch stream.
@@ -185,14 +192,15 @@ mpm_status mpm_merge_timed(const void* tokens, const int64_t* offsets, int32_t b
     if (stage_events == nullptr) return true;
     return cudaEventRecord(static_cast<cudaEvent_t>(stage_events[idx]), s) == cudaSuccess;
   };
-  const mpm::AffinityTile tile = algo == MPM_NN_TCGEN05 ? mpm::tc_tile() : mpm::simt_tile();
+  const bool sym = algo == MPM_NN_TCGEN05_SYM;
+  const mpm::AffinityTile tile = tc ? mpm::tc_tile(sym) : mpm::simt_tile();
   cudaError_t e = cudaSuccess;
   if (!mark(0)) return MPM_ERR_CUDA;
   e = mpm::launch_prep(tokens, offsets, batch, rows, dim, bf16, tile, ws, sms, s);
   if (e != cudaSuccess || !mark(1) || !mark(2)) return MPM_ERR_CUDA;
   if (rows > 0) {
-    e = algo == MPM_NN_TCGEN05 ? mpm::launch_affinity_tc(tokens, batch, rows, dim, ws, sms, s)
-                               : mpm::launch_affinity_simt(tokens, batch, dim, bf16, ws, sms, s);
+    e = tc ? mpm::launch_affinity_tc(tokens, batch, rows, dim, sym, ws, sms, s)
+           : mpm::launch_affinity_simt(tokens, batch, dim, bf16, ws, sms, s);
     if (e != cudaSuccess) return MPM_ERR_CUDA;
   }
   if (!mark(3) || !mark(4)) return MPM_ERR_CUDA;

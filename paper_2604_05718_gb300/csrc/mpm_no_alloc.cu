@@ -26,7 +26,7 @@
 
 #include <mutex>
 
-#include "../../include/mpm.h"
+#include "mpm.h"
 
 namespace {
 

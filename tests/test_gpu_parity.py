@@ -60,10 +60,11 @@ def merge_parity(mpm, batch, what: str, algo: str = "auto") -> ParityStats:
 RAGGED = [0, 1, 2, 3, 127, 128, 129, 255, 256, 257, 300, 1000]
 
 
+@pytest.mark.parametrize("algo", ["tcgen05_sym", "tcgen05"])
 @pytest.mark.parametrize("dim", [8, 64, 200, 384, 1024])
-def test_bf16_ragged_tcgen05(mpm, dim):
+def test_bf16_ragged_tcgen05(mpm, dim, algo):
     batch = make_custom(RAGGED, dim, "bf16", seed=dim)
-    st = merge_parity(mpm, batch, f"bf16 d={dim}")
+    st = merge_parity(mpm, batch, f"bf16 d={dim} {algo}", algo=algo)
     assert st.images == len(RAGGED)
 
 
@@ -82,8 +83,8 @@ def test_f32_ragged(mpm, dim):
     merge_parity(mpm, batch, f"f32 d={dim}")
 
 
-@pytest.mark.parametrize("dtype", ["bf16", "f32"])
-@pytest.mark.parametrize("algo", ["auto", "simt"])
+@pytest.mark.parametrize("dtype,algo", [("bf16", "auto"), ("bf16", "tcgen05"), ("bf16", "simt"),
+                                        ("f32", "auto"), ("f32", "simt")])
 def test_hand_examples_on_gpu(mpm, dtype, algo):
     """Every hand-worked example, packed into one ragged batch, zero-padded to 64 features."""
     exs = load_hand_examples()
@@ -104,8 +105,9 @@ def test_hand_examples_on_gpu(mpm, dtype, algo):
         np.testing.assert_array_equal(g["out"][o0:o1], want, err_msg=e.name)
 
 
-@pytest.mark.parametrize("dtype", ["bf16", "f32"])
-def test_exact_ties_duplicates_and_zero_rows(mpm, dtype):
+@pytest.mark.parametrize("dtype,algo", [("bf16", "tcgen05_sym"), ("bf16", "tcgen05"), ("bf16", "simt"),
+                                        ("f32", "simt")])
+def test_exact_ties_duplicates_and_zero_rows(mpm, dtype, algo):
     rng = np.random.default_rng(5)
     dim = 64
     same = np.tile(rng.standard_normal((1, dim)), (300, 1))                      # all identical
@@ -118,7 +120,7 @@ def test_exact_ties_duplicates_and_zero_rows(mpm, dtype):
     x = np.concatenate(parts, axis=0)
     offsets = np.concatenate([[0], np.cumsum([p.shape[0] for p in parts])]).astype(np.int64)
     t = torch.from_numpy(x.astype(np.float32)).to(DTYPES[dtype])
-    g = run_merge(mpm, t, offsets)
+    g = run_merge(mpm, t, offsets, algo)
     # Identical tokens: b(0) = 1, b(i >= 1) = 0, one pair.
     assert g["nn"][0] == 1 and np.all(g["nn"][1:300] == 0)
     assert g["out_offsets"][1] == 299
@@ -130,27 +132,31 @@ def test_exact_ties_duplicates_and_zero_rows(mpm, dtype):
     check_merge_batch(xs, offsets, g["nn"], g["map"], g["out"], g["out_offsets"], dtype, "ties")
 
 
-def test_large_dim_and_large_image(mpm):
+@pytest.mark.parametrize("algo", ["tcgen05_sym", "tcgen05"])
+def test_large_dim_and_large_image(mpm, algo):
     batch = make_custom([300, 77], 4096, "bf16", seed=41)
-    merge_parity(mpm, batch, "d=4096")
+    merge_parity(mpm, batch, "d=4096", algo=algo)
     big = make_custom([6000], 64, "bf16", seed=42, k=60)
-    merge_parity(mpm, big, "n=6000")
+    merge_parity(mpm, big, "n=6000", algo=algo)
 
 
 def test_tcgen05_and_simt_agree(mpm):
-    batch = make_custom([1000, 513, 64], 384, "bf16", seed=9)
-    a = run_merge(mpm, batch.tokens, batch.offsets, "tcgen05")
-    b = run_merge(mpm, batch.tokens, batch.offsets, "simt")
+    batch = make_custom([1000, 513, 64, 2300], 384, "bf16", seed=9)
+    runs = {algo: run_merge(mpm, batch.tokens, batch.offsets, algo) for algo in ("tcgen05", "tcgen05_sym", "simt")}
     res = [oracle.merge_image(batch.tokens[batch.offsets[k]:batch.offsets[k + 1]].double().numpy())
-           for k in range(3)]
+           for k in range(batch.batch)]
     decisive = np.concatenate([~r.nn.near_tie for r in res])
-    assert np.array_equal(a["nn"][decisive], b["nn"][decisive])
-    np.testing.assert_allclose(a["score"], b["score"], rtol=0, atol=1e-5)
+    for algo in ("tcgen05_sym", "simt"):
+        assert np.array_equal(runs["tcgen05"]["nn"][decisive], runs[algo]["nn"][decisive]), algo
+        np.testing.assert_allclose(runs["tcgen05"]["score"], runs[algo]["score"], rtol=0, atol=1e-5)
+    # Dense and symmetric tilings see the very same dot products: identical results.
+    assert np.array_equal(runs["tcgen05"]["nn"], runs["tcgen05_sym"]["nn"])
 
 
-def test_scores_are_cosines(mpm):
+@pytest.mark.parametrize("algo", ["tcgen05_sym", "tcgen05"])
+def test_scores_are_cosines(mpm, algo):
     batch = make_custom([500, 300], 256, "bf16", seed=3)
-    g = run_merge(mpm, batch.tokens, batch.offsets)
+    g = run_merge(mpm, batch.tokens, batch.offsets, algo)
     x = batch.tokens.double().numpy()
     for k in range(2):
         a0, a1 = batch.offsets[k], batch.offsets[k + 1]
