@@ -10,7 +10,9 @@ encoder blocks; it is not part of MPM and is not timed.
   python bench.py --impl reference ...   # the fp64 CPU oracle on host cores
 
 Timing: CUDA events on the launch stream bracket the two timed segments of
-every step (merge 1; merge 2 + compose + gather); L2 is flushed before every
+every step (merge 1; merge 2 + compose + gather).  A second timed loop adds
+events around every kernel for the per-kernel breakdown and the roofline
+(those events serialise the kernels, so the step time comes from the first); L2 is flushed before every
 step by writing and then reading a 256 MiB buffer; W untimed warm-up steps; barrier + synchronize on
 both sides; the max over ranks is reported.  Each rank processes its own
 batch (images are independent: replicas, weak scaling, no collective on the
@@ -361,7 +363,9 @@ def run_mpm(args):
             self.k2 = new_events(8)        # merge 2 kernels
             self.cg = new_events(2)        # between compose and gather
 
-    def step(ev: StepEvents, host_in=None, host_out=None):
+    def step(ev: StepEvents, host_in=None, host_out=None, per_kernel=False):
+        """One step; per_kernel adds CUDA events between the kernels (which
+        serialises them, so the step time is taken without them)."""
         # Evict the L2: write 256 MiB, then read it back so that the lines left
         # behind are clean (no write-back lands on the first timed kernel).
         flush.fill_(1)
@@ -370,20 +374,25 @@ def run_mpm(args):
         if host_in is not None:
             x0.copy_(host_in[0], non_blocking=True)
             off0.copy_(host_in[1], non_blocking=True)
-        mpm.merge(x0, off0, workspace=ws, out_tokens=x1, out_offsets=off1, out_map=m1, stage_events=ev.k1)
+        mpm.merge(x0, off0, workspace=ws, out_tokens=x1, out_offsets=off1, out_map=m1,
+                  stage_events=ev.k1 if per_kernel else None)
         ev.seg[1].record(stream)
         if two:
             x1n[:t1] = apply_noise(x1[:t1], noise)
         ev.seg[2].record(stream)
         if two:
-            mpm.merge(x1n, off1, workspace=ws, out_tokens=x2, out_offsets=off2, out_map=m2, stage_events=ev.k2)
+            mpm.merge(x1n, off1, workspace=ws, out_tokens=x2, out_offsets=off2, out_map=m2,
+                      stage_events=ev.k2 if per_kernel else None)
             mpm.compose_maps(m1, off0, m2, off1, out=rstar)
-            ev.cg[0].record(stream)
+            if per_kernel:
+                ev.cg[0].record(stream)
             mpm.unmerge_gather(x2, off2, rstar, off0, out=up)
         else:
-            ev.cg[0].record(stream)
+            if per_kernel:
+                ev.cg[0].record(stream)
             mpm.unmerge_gather(x1, off1, m1, off0, out=up)
-        ev.cg[1].record(stream)
+        if per_kernel:
+            ev.cg[1].record(stream)
         if host_out is not None:
             host_out.copy_(up, non_blocking=True)
         ev.seg[3].record(stream)
@@ -421,9 +430,19 @@ def run_mpm(args):
     off2_h = off2.cpu().numpy() if two else off1_h
     assert mpm.device_status(ws) == 0, "device status reported an error in the timed loop"
 
+    # Second timed loop, same steps with CUDA events around every kernel: the
+    # per-kernel durations for the roofline and the breakdown.
+    kevents = [StepEvents() for _ in range(args.steps)]
+    barrier()
+    for ev in kevents:
+        step(ev, per_kernel=True)
+    barrier()
+    ms_with_kernel_events = max_over_ranks(statistics.mean(
+        [ev.seg[0].elapsed_time(ev.seg[1]) + ev.seg[2].elapsed_time(ev.seg[3]) for ev in kevents]))
+
     # Per-kernel durations inside the timed region.
     def kernel_ms(key, k):
-        return [getattr(ev, key)[2 * k].elapsed_time(getattr(ev, key)[2 * k + 1]) for ev in events]
+        return [getattr(ev, key)[2 * k].elapsed_time(getattr(ev, key)[2 * k + 1]) for ev in kevents]
 
     names = ["prep", "affinity", "mutual_scan", "pair_average"]
     kern = {}
@@ -431,7 +450,7 @@ def run_mpm(args):
         kern[f"{nm}_1_us"] = 1e3 * statistics.mean(kernel_ms("k1", k))
         if two:
             kern[f"{nm}_2_us"] = 1e3 * statistics.mean(kernel_ms("k2", k))
-    cg = [ev.cg[0].elapsed_time(ev.cg[1]) for ev in events]
+    cg = [ev.cg[0].elapsed_time(ev.cg[1]) for ev in kevents]
     kern["gather_us"] = 1e3 * statistics.mean(cg)
 
     peaks, peak_kind = load_peaks()
@@ -526,6 +545,7 @@ def run_mpm(args):
             "roofline": roofline,
             "hbm_kernels": hbm_kernels,
             "kernels_us": kern,
+            "ms_per_step_with_kernel_events": ms_with_kernel_events,
             "cpu_baseline": cpu_base,
             "e2e": e2e,
             "clocks": clk,

@@ -23,6 +23,7 @@ __device__ __forceinline__ float load_elem(const uint8_t* tokens, int64_t row, i
 template <bool BF16>
 __global__ void __launch_bounds__(kThreads) affinity_simt_kernel(const uint8_t* __restrict__ tokens, int batch,
                                                                  int dim, Workspace ws) {
+  wait_for_previous_grid();
   __shared__ __align__(16) float As[BK][BM + 4];
   __shared__ __align__(16) float Bs[BK][BN + 4];
   __shared__ float scale[BN];
@@ -105,12 +106,9 @@ AffinityTile simt_tile() { return {BM, BN, false}; }
 cudaError_t launch_affinity_simt(const void* tokens, int batch, int dim, bool bf16, const Workspace& ws,
                                  int num_sms, cudaStream_t stream) {
   const int grid = (num_sms > 0 ? num_sms : 1) * 4;
-  if (bf16) {
-    affinity_simt_kernel<true><<<grid, kThreads, 0, stream>>>(static_cast<const uint8_t*>(tokens), batch, dim, ws);
-  } else {
-    affinity_simt_kernel<false><<<grid, kThreads, 0, stream>>>(static_cast<const uint8_t*>(tokens), batch, dim, ws);
-  }
-  return cudaGetLastError();
+  const uint8_t* t = static_cast<const uint8_t*>(tokens);
+  if (bf16) return launch_dependent(affinity_simt_kernel<true>, dim3(grid), dim3(kThreads), 0, stream, t, batch, dim, ws);
+  return launch_dependent(affinity_simt_kernel<false>, dim3(grid), dim3(kThreads), 0, stream, t, batch, dim, ws);
 }
 
 }  // namespace mpm

@@ -63,6 +63,7 @@ constexpr int EPI_COLS = BN / (EPI_WARPS / 4);  // columns read by one epilogue 
 constexpr int THREADS = (2 + EPI_WARPS) * 32;
 constexpr uint32_t TMEM_COLS = 2 * BN;         // double-buffered accumulator
 constexpr uint32_t IDESC = ptx::idesc_bf16_f32(BM, BN);
+constexpr uint32_t IDESC_HALF = ptx::idesc_bf16_f32(BM, BN / 2);  // upper 128-column block only
 constexpr uint64_t WAIT_LIMIT_NS = 2000000000ull;  // 2 s per wait
 
 struct Control {
@@ -86,6 +87,8 @@ struct Item {
   int n;         // tokens in the image
   int row0;      // first local row of the tile (row block I = row0 / 128)
   int col0;      // first local column of the tile (column blocks 2T, 2T+1 with T = col0 / 256)
+  bool upper_only;  // symmetric mode: block 2T lies below the diagonal, so only
+                    // block 2T+1 (the diagonal block) is loaded and multiplied
 };
 
 template <bool SYM>
@@ -99,6 +102,7 @@ __device__ __forceinline__ Item decode_item(const Workspace& ws, int batch, int6
   if (!SYM) {
     it.row0 = static_cast<int>(local / c) * BM;
     it.col0 = static_cast<int>(local % c) * BN;
+    it.upper_only = false;
     return it;
   }
   // Symmetric tiling (see affinity_tiles): row blocks 2m and 2m+1 start at
@@ -116,6 +120,7 @@ __device__ __forceinline__ Item decode_item(const Workspace& ws, int batch, int6
   if (local >= per) local -= per;
   it.row0 = static_cast<int>(blk) * BM;
   it.col0 = static_cast<int>(lo + local) * BN;
+  it.upper_only = it.col0 / BM < blk;
   return it;
 }
 
@@ -186,6 +191,7 @@ template <bool SYM>
 __global__ void __launch_bounds__(THREADS, 1)
     affinity_tc_kernel(const __grid_constant__ CUtensorMap tmap, int batch, int ksteps, Workspace ws) {
   extern __shared__ uint8_t smem_raw[];
+  wait_for_previous_grid();
   uint8_t* smem = smem_raw + ((1024u - (ptx::smem_addr(smem_raw) & 1023u)) & 1023u);
   uint8_t* stages = smem;
   float* scale = reinterpret_cast<float*>(smem + STAGES * STAGE_BYTES);  // [2][BN]
@@ -242,9 +248,9 @@ __global__ void __launch_bounds__(THREADS, 1)
           }
           uint8_t* sa = stages + stage * STAGE_BYTES;
           uint8_t* sb = sa + A_BYTES;
-          ptx::mbar_arrive_expect_tx(&ctl->full[stage], STAGE_BYTES);
+          ptx::mbar_arrive_expect_tx(&ctl->full[stage], it.upper_only ? A_BYTES + B_BYTES / 2 : STAGE_BYTES);
           ptx::tma_load_2d(sa, &tmap, &ctl->full[stage], kb * BK, arow);
-          ptx::tma_load_2d(sb, &tmap, &ctl->full[stage], kb * BK, brow);
+          if (!it.upper_only) ptx::tma_load_2d(sb, &tmap, &ctl->full[stage], kb * BK, brow);
           ptx::tma_load_2d(sb + B_BYTES / 2, &tmap, &ctl->full[stage], kb * BK, brow + TMA_ROWS);
           issued |= 1 << stage;
           issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
@@ -268,12 +274,17 @@ __global__ void __launch_bounds__(THREADS, 1)
       uint32_t phase = 0, acc_phase = 0;
       bool ok = true;
       for (int64_t w = blockIdx.x; ok && w < total; w += gridDim.x) {
+        // Tiles whose lower 128-column block is below the diagonal multiply
+        // only the upper block (N = 128) into the upper half of the accumulator.
+        const bool upper_only = SYM && decode_item<SYM>(ws, batch, w).upper_only;
+        const uint32_t idesc = upper_only ? IDESC_HALF : IDESC;
+        const uint32_t b_off = upper_only ? B_BYTES / 2 : 0;
         if (!ptx::mbar_wait(&ctl->acc_empty[acc], acc_phase ^ 1u, abort_flag, WAIT_LIMIT_NS)) {
           fail(ctl, ws.status, 2);
           break;
         }
         ptx::tc_fence_after_sync();
-        const uint32_t d_tmem = tmem + static_cast<uint32_t>(acc * BN);
+        const uint32_t d_tmem = tmem + static_cast<uint32_t>(acc * BN) + (upper_only ? BN / 2 : 0);
         for (int kb = 0; kb < ksteps; ++kb) {
           if (!ptx::mbar_wait(&ctl->full[stage], phase, abort_flag, WAIT_LIMIT_NS)) {
             fail(ctl, ws.status, 3);
@@ -282,12 +293,12 @@ __global__ void __launch_bounds__(THREADS, 1)
           }
           ptx::tc_fence_after_sync();
           const uint32_t a_addr = ptx::smem_addr(stages + stage * STAGE_BYTES);
-          const uint32_t b_addr = a_addr + A_BYTES;
+          const uint32_t b_addr = a_addr + A_BYTES + b_off;
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k) {
             // Advancing the start address by 32 bytes steps K by 16 inside
             // the 128-byte swizzled row.
-            ptx::mma_bf16(d_tmem, ptx::sdesc_k_sw128(a_addr + k * 32), ptx::sdesc_k_sw128(b_addr + k * 32), IDESC,
+            ptx::mma_bf16(d_tmem, ptx::sdesc_k_sw128(a_addr + k * 32), ptx::sdesc_k_sw128(b_addr + k * 32), idesc,
                           (kb | k) != 0 ? 1u : 0u);
           }
           ptx::mma_commit(&ctl->empty[stage]);
@@ -456,13 +467,13 @@ cudaError_t launch_affinity_tc(const void* tokens, int batch, int64_t rows, int 
   if (symmetric) {
     e = ensure_smem_attr<true>();
     if (e != cudaSuccess) return e;
-    affinity_tc_kernel<true><<<grid, THREADS, SMEM_BYTES, stream>>>(map, batch, ksteps, ws);
-  } else {
-    e = ensure_smem_attr<false>();
-    if (e != cudaSuccess) return e;
-    affinity_tc_kernel<false><<<grid, THREADS, SMEM_BYTES, stream>>>(map, batch, ksteps, ws);
+    return launch_dependent(affinity_tc_kernel<true>, dim3(grid), dim3(THREADS), SMEM_BYTES, stream, map, batch,
+                            ksteps, ws);
   }
-  return cudaGetLastError();
+  e = ensure_smem_attr<false>();
+  if (e != cudaSuccess) return e;
+  return launch_dependent(affinity_tc_kernel<false>, dim3(grid), dim3(THREADS), SMEM_BYTES, stream, map, batch, ksteps,
+                          ws);
 }
 
 }  // namespace mpm

@@ -41,6 +41,7 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(const uint8_t* __restric
                                                         int batch, int64_t rows, int row_bytes,
                                                         bool bf16, AffinityTile tile,
                                                         Workspace ws) {
+  wait_for_previous_grid();
   if (blockIdx.x == 0) {
     __shared__ int64_t sh[32];
     __shared__ int bad;
@@ -140,6 +141,7 @@ constexpr int kScanThreads = 1024;
 __global__ void __launch_bounds__(kScanThreads) mutual_compact_kernel(int batch, Workspace ws,
                                                                       int32_t* __restrict__ out_map,
                                                                       int64_t* __restrict__ out_offsets) {
+  wait_for_previous_grid();
   __shared__ int32_t sh[32];
   __shared__ int64_t sh64[32];
   __shared__ int is_last;
@@ -200,6 +202,7 @@ __global__ void __launch_bounds__(kThreads) pair_average_kernel(const uint8_t* _
                                                                 int batch, int64_t rows, int row_bytes,
                                                                 bool bf16, Workspace ws,
                                                                 const int64_t* __restrict__ out_offsets) {
+  wait_for_previous_grid();
   const int lane = threadIdx.x & 31;
   const int64_t warp = (static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x) >> 5;
   const int64_t nwarps = (static_cast<int64_t>(gridDim.x) * kThreads) >> 5;
@@ -257,6 +260,7 @@ __global__ void __launch_bounds__(kThreads) pair_average_kernel(const uint8_t* _
 // ---------------------------------------------------------------------------
 __global__ void decode_nn_kernel(int batch, int64_t rows, Workspace ws, int32_t* __restrict__ nn,
                                  float* __restrict__ score) {
+  wait_for_previous_grid();
   const int64_t used = ws.soff[batch];
   for (int64_t g = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; g < used;
        g += static_cast<int64_t>(gridDim.x) * blockDim.x) {
@@ -275,6 +279,7 @@ __global__ void compose_kernel(const int32_t* map1, const int64_t* __restrict__ 
                                int64_t rows0, const int32_t* __restrict__ map2,
                                const int64_t* __restrict__ off1, int64_t rows1, int batch,
                                int32_t* out, int32_t* status) {
+  wait_for_previous_grid();
   const int64_t used = clamp64(off0[batch], 0, rows0);
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   for (int64_t p = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; p < used; p += stride) {
@@ -303,6 +308,7 @@ __global__ void __launch_bounds__(kThreads) gather_kernel(const uint8_t* __restr
                                                           const int64_t* __restrict__ goff,
                                                           int64_t grid_rows, int batch, int row_bytes,
                                                           uint8_t* __restrict__ out, int32_t* status) {
+  wait_for_previous_grid();
   const int lane = threadIdx.x & 31;
   const int64_t warp = (static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x) >> 5;
   const int64_t nwarps = (static_cast<int64_t>(gridDim.x) * kThreads) >> 5;
@@ -342,40 +348,37 @@ cudaError_t launch_prep(const void* tokens, const int64_t* offsets, int batch, i
                         bool bf16, AffinityTile tile, const Workspace& ws, int num_sms,
                         cudaStream_t stream) {
   const int row_bytes = dim * (bf16 ? 2 : 4);
-  prep_kernel<<<grid_for(num_sms, 8), kThreads, 0, stream>>>(
-      static_cast<const uint8_t*>(tokens), offsets, batch, rows, row_bytes, bf16, tile, ws);
-  return cudaGetLastError();
+  return launch_dependent(prep_kernel, dim3(grid_for(num_sms, 8)), dim3(kThreads), 0, stream,
+                          static_cast<const uint8_t*>(tokens), offsets, batch, rows, row_bytes, bf16, tile, ws);
 }
 
 cudaError_t launch_mutual_compact(int batch, const Workspace& ws, int32_t* out_map,
                                   int64_t* out_offsets, cudaStream_t stream) {
-  mutual_compact_kernel<<<batch, kScanThreads, 0, stream>>>(batch, ws, out_map, out_offsets);
-  return cudaGetLastError();
+  return launch_dependent(mutual_compact_kernel, dim3(batch), dim3(kScanThreads), 0, stream, batch, ws, out_map,
+                          out_offsets);
 }
 
 cudaError_t launch_pair_average(const void* tokens, void* out_tokens, int batch, int64_t rows,
                                 int dim, bool bf16, const Workspace& ws,
                                 const int64_t* out_offsets, int num_sms, cudaStream_t stream) {
   const int row_bytes = dim * (bf16 ? 2 : 4);
-  pair_average_kernel<1, 4><<<grid_for(num_sms, 8), kThreads, 0, stream>>>(
-      static_cast<const uint8_t*>(tokens), static_cast<uint8_t*>(out_tokens), batch, rows,
-      row_bytes, bf16, ws, out_offsets);
-  return cudaGetLastError();
+  return launch_dependent(pair_average_kernel<1, 4>, dim3(grid_for(num_sms, 8)), dim3(kThreads), 0, stream,
+                          static_cast<const uint8_t*>(tokens), static_cast<uint8_t*>(out_tokens), batch, rows,
+                          row_bytes, bf16, ws, out_offsets);
 }
 
 cudaError_t launch_decode_nn(int batch, int64_t rows, const Workspace& ws, int32_t* out_nn,
                              float* out_score, int num_sms, cudaStream_t stream) {
   (void)rows;
-  decode_nn_kernel<<<grid_for(num_sms, 4), kThreads, 0, stream>>>(batch, rows, ws, out_nn, out_score);
-  return cudaGetLastError();
+  return launch_dependent(decode_nn_kernel, dim3(grid_for(num_sms, 4)), dim3(kThreads), 0, stream, batch, rows, ws,
+                          out_nn, out_score);
 }
 
 cudaError_t launch_compose(const int32_t* map1, const int64_t* off0, int64_t rows0,
                            const int32_t* map2, const int64_t* off1, int64_t rows1, int batch,
                            int32_t* out, int32_t* status, int num_sms, cudaStream_t stream) {
-  compose_kernel<<<grid_for(num_sms, 4), kThreads, 0, stream>>>(map1, off0, rows0, map2, off1,
-                                                                  rows1, batch, out, status);
-  return cudaGetLastError();
+  return launch_dependent(compose_kernel, dim3(grid_for(num_sms, 4)), dim3(kThreads), 0, stream, map1, off0, rows0,
+                          map2, off1, rows1, batch, out, status);
 }
 
 cudaError_t launch_gather(const void* merged, const int64_t* moff, int64_t merged_rows,
@@ -383,10 +386,9 @@ cudaError_t launch_gather(const void* merged, const int64_t* moff, int64_t merge
                           int dim, bool bf16, void* out, int32_t* status, int num_sms,
                           cudaStream_t stream) {
   const int row_bytes = dim * (bf16 ? 2 : 4);
-  gather_kernel<4><<<grid_for(num_sms, 8), kThreads, 0, stream>>>(
-      static_cast<const uint8_t*>(merged), moff, merged_rows, map, goff, grid_rows, batch,
-      row_bytes, static_cast<uint8_t*>(out), status);
-  return cudaGetLastError();
+  return launch_dependent(gather_kernel<4>, dim3(grid_for(num_sms, 8)), dim3(kThreads), 0, stream,
+                          static_cast<const uint8_t*>(merged), moff, merged_rows, map, goff, grid_rows, batch,
+                          row_bytes, static_cast<uint8_t*>(out), status);
 }
 
 }  // namespace mpm
