@@ -73,11 +73,13 @@ typedef enum mpm_status {
 
 /* Which kernel computes the nearest neighbours (Eq. 1 + arg max). */
 typedef enum mpm_nn_algo {
-  MPM_NN_AUTO = 0,        /* MPM_NN_TCGEN05_SYM for bf16, MPM_NN_SIMT for fp32 */
-  MPM_NN_SIMT = 1,        /* CUDA-core fp32 FMA tiles (any dtype) */
-  MPM_NN_TCGEN05 = 2,     /* TMA + tcgen05 MMA into TMEM, every tile of X X^T (bf16) */
-  MPM_NN_TCGEN05_SYM = 3  /* as above, tiles on or above the diagonal only, each
-                             feeding both its rows and its columns (bf16) */
+  MPM_NN_AUTO = 0,         /* MPM_NN_TCGEN05_PAIR for bf16, MPM_NN_SIMT for fp32 */
+  MPM_NN_SIMT = 1,         /* CUDA-core fp32 FMA tiles (any dtype) */
+  MPM_NN_TCGEN05 = 2,      /* TMA + tcgen05 MMA into TMEM, every tile of X X^T (bf16) */
+  MPM_NN_TCGEN05_SYM = 3,  /* as above, tiles on or above the diagonal only, each
+                              feeding both its rows and its columns (bf16) */
+  MPM_NN_TCGEN05_PAIR = 4  /* symmetric, 256 x 256 tiles on SM pairs with
+                              tcgen05.mma.cta_group::2 (bf16) */
 } mpm_nn_algo;
 
 /* Version of this ABI (MPM_ABI_VERSION). */

@@ -1,0 +1,529 @@
+// Symmetric affinity + arg max on SM pairs (bf16): the default kernel for
+// Eq. 1 and Algorithm 1 step 3.
+//
+// Same arithmetic as affinity_tc.cu (raw bf16 dot products accumulated in
+// fp32 in tensor memory, scaled in fp32 by 1/max(|x|, 1e-12) in the
+// epilogue, packed (score, lowest index) keys merged with atomicMax), with
+// two changes in how the work is laid out:
+//
+//  * A cluster of two CTAs (an SM pair) computes a 256 x 256 tile of
+//    G = X X^T with tcgen05.mma.cta_group::2 (M = 256, N = 256).  CTA r holds
+//    tile rows [128r, 128r + 128) of A and tile columns [128r, 128r + 128) of
+//    B in its own shared memory, and receives its 128 rows x 256 columns of
+//    the accumulator in its own tensor memory.  Each SM therefore stages 32
+//    KiB per 64-feature step instead of 48 KiB, which leaves room for six
+//    stages and cuts the shared-memory traffic of the tensor cores by a third.
+//  * Tiles are the 256 x 256 blocks on or above the diagonal of each image's
+//    G, R(R + 1) / 2 of them for R = ceil(N_b / 256).  Within a tile, every
+//    128-column block above a thread's 128-row block also yields column
+//    candidates (row j scores row i by G_ij / |x_i|), as in affinity_tc.cu's
+//    symmetric mode; the block below the diagonal of a diagonal tile is
+//    skipped.
+//
+// Roles per CTA (18 warps): warp 0 loads its CTA's A and B slices with TMA
+// and reports the bytes to the leader CTA's barrier; in the leader, warp 1
+// allocates tensor memory (jointly with the peer) and issues the MMAs, whose
+// completion is multicast to both CTAs; warps 2-17 of each CTA read their own
+// tensor memory in 32 x 64 slices.  Every wait is bounded; on expiry the
+// kernel records MPM_ERR_DEVICE_TIMEOUT and unwinds.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <math.h>
+
+#include <atomic>
+
+#include "mpm.h"
+#include "common.cuh"
+#include "ptx.cuh"
+
+namespace mpm {
+namespace {
+
+constexpr int TILE = 256;                      // tile rows and columns
+constexpr int HALF = 128;                      // rows of A / B per CTA
+constexpr int BK = 64;
+constexpr int STAGES = 6;
+constexpr int SLICE_BYTES = HALF * BK * 2;     // 16 KiB
+constexpr int STAGE_BYTES = 2 * SLICE_BYTES;   // A slice + B slice of this CTA
+constexpr int EPI_WARPS = 16;
+constexpr int EPI_COLS = TILE / (EPI_WARPS / 4);
+constexpr int THREADS = (2 + EPI_WARPS) * 32;
+constexpr uint32_t TMEM_COLS = 2 * TILE;
+constexpr uint32_t IDESC = ptx::idesc_bf16_f32(2 * HALF, TILE);
+constexpr uint64_t WAIT_LIMIT_NS = 2000000000ull;
+constexpr int kMaxItems = 160;
+constexpr int kMaxStagedImages = 511;  // plan and offsets staged in shared memory up to this batch
+
+struct Control {
+  uint64_t full[STAGES];        // leader: all four slices of stage s landed
+  uint64_t empty[STAGES];       // both: MMAs reading stage s completed
+  uint64_t acc_full[2];         // both: accumulator a complete
+  uint64_t acc_empty[2];        // leader: both CTAs finished reading accumulator a
+  uint64_t scale_ready[2];      // local: column scales of accumulator a written
+  uint64_t drain;               // leader: all MMAs completed
+  unsigned long long colkey[2][TILE];
+  int colcount[2];
+  uint32_t tmem_base;
+  int abort_flag;
+};
+
+struct Item {
+  int64_t base;
+  int n;
+  int row0;  // first local row of the tile (a multiple of 256)
+  int col0;  // first local column of the tile (a multiple of 256)
+};
+
+constexpr size_t SMEM_BYTES = 1024 + static_cast<size_t>(STAGES) * STAGE_BYTES + 2 * TILE * sizeof(float) +
+                              sizeof(Control) + 16 + kMaxItems * sizeof(Item) +
+                              2 * (kMaxStagedImages + 1) * sizeof(int64_t);
+
+// Item w of the launch: image by the plan, then the upper-triangle tile (I, J),
+// J >= I, numbered row by row: row I starts at P(I) = I R - I (I - 1) / 2.
+// `plan` and `soff` are the work plan and sanitised offsets, in shared or
+// global memory.
+__device__ __forceinline__ Item decode_pair_item(const int64_t* plan, const int64_t* soff, int batch, int64_t w) {
+  int lo_b = 0, hi_b = batch - 1;
+  while (lo_b < hi_b) {
+    const int mid = (lo_b + hi_b + 1) >> 1;
+    if (plan[mid] <= w) lo_b = mid; else hi_b = mid - 1;
+  }
+  const int b = lo_b;
+  int64_t local = w - plan[b];
+  Item it;
+  it.base = soff[b];
+  it.n = static_cast<int>(soff[b + 1] - it.base);
+  const int64_t r = (it.n + TILE - 1) / TILE;
+  int64_t lo = 0, hi = r - 1;
+  while (lo < hi) {
+    const int64_t mid = (lo + hi + 1) / 2;
+    if (mid * r - mid * (mid - 1) / 2 <= local) lo = mid; else hi = mid - 1;
+  }
+  local -= lo * r - lo * (lo - 1) / 2;
+  it.row0 = static_cast<int>(lo) * TILE;
+  it.col0 = static_cast<int>(lo + local) * TILE;
+  return it;
+}
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t cluster_id() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%clusterid.x;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t cluster_count() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%nclusterid.x;" : "=r"(r));
+  return r;
+}
+// Address of the same shared-memory location in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t map_to_rank(uint32_t saddr, uint32_t rank) {
+  uint32_t out;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(out) : "r"(saddr), "r"(rank));
+  return out;
+}
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void remote_arrive(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+// TMA tile load into this CTA's shared memory whose completion is counted on
+// an mbarrier of either CTA of the pair.
+__device__ __forceinline__ void tma_load_2d_pair(void* dst, const CUtensorMap* map, uint32_t bar_cluster, int32_t x,
+                                                 int32_t y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], "
+      "[%2];" ::"r"(ptx::smem_addr(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster), "r"(x), "r"(y)
+      : "memory");
+}
+__device__ __forceinline__ void mma_pair(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                         uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// Arrives on the barrier at this offset in both CTAs once the MMAs issued so
+// far completed.
+__device__ __forceinline__ void commit_both(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+          ptx::smem_addr(bar)),
+      "h"(static_cast<uint16_t>(3))
+      : "memory");
+}
+__device__ __forceinline__ void commit_local(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(ptx::smem_addr(bar))
+               : "memory");
+}
+
+__device__ __forceinline__ int float_order_s32(float x) {
+  const int b = __float_as_int(x);
+  return b ^ ((b >> 31) & 0x7FFFFFFF);
+}
+
+__device__ __forceinline__ void fail(Control* ctl, int32_t* status, int32_t role) {
+  ctl->abort_flag = 1;
+  report(status, MPM_ERR_DEVICE_TIMEOUT, role);
+}
+
+// One 32-column chunk for the thread's row (see affinity_tc.cu's
+// epilogue_chunk for the reasoning; the arithmetic is the same).
+template <bool DIAG, bool COL>
+__device__ __forceinline__ void chunk(const uint32_t (&v)[32], const float* sc, int c, int jd, float& best, int& bj,
+                                      float inv_i, int lane, int row_base, int n, int col0,
+                                      unsigned long long* colkey) {
+#pragma unroll
+  for (int k = 0; k < 32; k += 4) {
+    const float4 s4 = *reinterpret_cast<const float4*>(sc + c + k);
+    const float sv[4] = {s4.x, s4.y, s4.z, s4.w};
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const float s = __uint_as_float(v[k + u]) * sv[u];
+      if (s > best && (!DIAG || c + k + u != jd)) {
+        best = s;
+        bj = c + k + u;
+      }
+    }
+  }
+  if (COL) {
+    int top = 0;
+    uint32_t lanes = 0;
+#pragma unroll
+    for (int k = 0; k < 32; ++k) {
+      const int key = float_order_s32(__fmaf_rn(__uint_as_float(v[k]), inv_i, 0.0f));
+      const int m = __reduce_max_sync(0xFFFFFFFFu, key);
+      const uint32_t ball = __ballot_sync(0xFFFFFFFFu, key == m);
+      if (lane == k) {
+        top = m;
+        lanes = ball;
+      }
+    }
+    const int winner = row_base + __ffs(static_cast<int>(lanes)) - 1;
+    if (winner < n && col0 + c + lane < n) {
+      const uint32_t hi = static_cast<uint32_t>(top) ^ 0x80000000u;
+      atomicMax(colkey + c + lane, (static_cast<unsigned long long>(hi) << 32) |
+                                       static_cast<unsigned long long>(0xFFFFFFFFu - static_cast<uint32_t>(winner)));
+    }
+  }
+}
+
+__global__ void __launch_bounds__(THREADS, 1)
+    affinity_pair_kernel(const __grid_constant__ CUtensorMap tmap, int batch, int ksteps, Workspace ws) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = smem_raw + ((1024u - (ptx::smem_addr(smem_raw) & 1023u)) & 1023u);
+  uint8_t* stages = smem;
+  float* scale = reinterpret_cast<float*>(smem + STAGES * STAGE_BYTES);  // [2][TILE]
+  Control* ctl = reinterpret_cast<Control*>(smem + STAGES * STAGE_BYTES + 2 * TILE * sizeof(float));
+  Item* items = reinterpret_cast<Item*>((reinterpret_cast<uintptr_t>(ctl + 1) + 15) & ~static_cast<uintptr_t>(15));
+  int64_t* plan_s = reinterpret_cast<int64_t*>(items + kMaxItems);
+  int64_t* soff_s = plan_s + kMaxStagedImages + 1;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_rank();
+  const bool leader = rank == 0;
+  const int64_t clusters = cluster_count();
+  const int64_t cid = cluster_id();
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      ptx::mbar_init(&ctl->full[s], 1);
+      ptx::mbar_init(&ctl->empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      ptx::mbar_init(&ctl->acc_full[a], 1);
+      // Leader's threads arrive one by one, the peer's warps once each.
+      ptx::mbar_init(&ctl->acc_empty[a], EPI_WARPS * 32 + EPI_WARPS);
+      ptx::mbar_init(&ctl->scale_ready[a], EPI_WARPS * 32);
+      ctl->colcount[a] = 0;
+    }
+    ptx::mbar_init(&ctl->drain, 1);
+    ctl->abort_flag = 0;
+    ptx::fence_barrier_init();
+    ptx::prefetch_tensor_map(&tmap);
+  }
+  for (int e = threadIdx.x; e < 2 * TILE; e += THREADS) (&ctl->colkey[0][0])[e] = 0ull;
+  if (warp == 1) {
+    // Both CTAs of the pair take part in the joint allocation.
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     ptx::smem_addr(&ctl->tmem_base)),
+                 "r"(TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+  }
+  ptx::tc_fence_before_sync();
+  __syncthreads();
+  cluster_sync();  // barriers of both CTAs exist before any remote signal
+  ptx::tc_fence_after_sync();
+  const uint32_t tmem = ctl->tmem_base;
+
+  // Everything above touches no data of earlier kernels; from here on the
+  // work plan, offsets and norms written by the prep kernel are read.
+  wait_for_previous_grid();
+  const bool staged = batch <= kMaxStagedImages;
+  if (staged) {
+    for (int e = threadIdx.x; e <= batch; e += THREADS) {
+      plan_s[e] = ws.plan[e];
+      soff_s[e] = ws.soff[e];
+    }
+    __syncthreads();
+  }
+  const int64_t* plan = staged ? plan_s : ws.plan;
+  const int64_t* soff = staged ? soff_s : ws.soff;
+  const int64_t total = plan[batch];
+  const int64_t count = total > cid ? (total - 1 - cid) / clusters + 1 : 0;
+  for (int64_t k = threadIdx.x; k < count && k < kMaxItems; k += THREADS)
+    items[k] = decode_pair_item(plan, soff, batch, cid + k * clusters);
+  __syncthreads();
+  auto item = [&](int64_t k) -> Item {
+    return k < kMaxItems ? items[k] : decode_pair_item(plan, soff, batch, cid + k * clusters);
+  };
+  volatile int* abort_flag = &ctl->abort_flag;
+
+  if (warp == 0) {
+    // ---------------- TMA producer (both CTAs) ----------------
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int issued = 0;
+      uint32_t issued_phase = 0;
+      bool ok = true;
+      for (int64_t k = 0; ok && k < count; ++k) {
+        const Item it = item(k);
+        const int32_t arow = static_cast<int32_t>(it.base + it.row0 + HALF * rank);
+        const int32_t brow = static_cast<int32_t>(it.base + it.col0 + HALF * rank);
+        for (int kb = 0; kb < ksteps; ++kb) {
+          if (!ptx::mbar_wait(&ctl->empty[stage], phase ^ 1u, abort_flag, WAIT_LIMIT_NS)) {
+            fail(ctl, ws.status, 11);
+            ok = false;
+            break;
+          }
+          uint8_t* sa = stages + stage * STAGE_BYTES;
+          const uint32_t full_leader = map_to_rank(ptx::smem_addr(&ctl->full[stage]), 0);
+          if (leader) ptx::mbar_arrive_expect_tx(&ctl->full[stage], 2 * STAGE_BYTES);
+          tma_load_2d_pair(sa, &tmap, full_leader, kb * BK, arow);
+          tma_load_2d_pair(sa + SLICE_BYTES, &tmap, full_leader, kb * BK, brow);
+          issued |= 1 << stage;
+          issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      if (!ok && leader) {
+        for (int s = 0; s < STAGES; ++s)
+          if (issued & (1 << s)) ptx::mbar_wait(&ctl->full[s], (issued_phase >> s) & 1u, nullptr, WAIT_LIMIT_NS);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    // ---------------- MMA issuer (leader) ----------------
+    if (leader && lane == 0) {
+      int stage = 0, acc = 0;
+      uint32_t phase = 0, acc_phase = 0;
+      bool ok = true;
+      for (int64_t k = 0; ok && k < count; ++k) {
+        if (!ptx::mbar_wait(&ctl->acc_empty[acc], acc_phase ^ 1u, abort_flag, WAIT_LIMIT_NS)) {
+          fail(ctl, ws.status, 12);
+          break;
+        }
+        ptx::tc_fence_after_sync();
+        const uint32_t d_tmem = tmem + static_cast<uint32_t>(acc * TILE);
+        for (int kb = 0; kb < ksteps; ++kb) {
+          if (!ptx::mbar_wait(&ctl->full[stage], phase, abort_flag, WAIT_LIMIT_NS)) {
+            fail(ctl, ws.status, 13);
+            ok = false;
+            break;
+          }
+          ptx::tc_fence_after_sync();
+          const uint32_t a_addr = ptx::smem_addr(stages + stage * STAGE_BYTES);
+          const uint32_t b_addr = a_addr + SLICE_BYTES;
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk)
+            mma_pair(d_tmem, ptx::sdesc_k_sw128(a_addr + kk * 32), ptx::sdesc_k_sw128(b_addr + kk * 32), IDESC,
+                     (kb | kk) != 0 ? 1u : 0u);
+          commit_both(&ctl->empty[stage]);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        commit_both(&ctl->acc_full[acc]);
+        if (++acc == 2) {
+          acc = 0;
+          acc_phase ^= 1u;
+        }
+      }
+      commit_local(&ctl->drain);
+      ptx::mbar_wait(&ctl->drain, 0, nullptr, WAIT_LIMIT_NS);
+    }
+    __syncwarp();
+  } else {
+    // ---------------- epilogue (both CTAs) ----------------
+    const int ew = warp - 2;
+    const int q = warp & 3;
+    const int quarter = ew >> 2;
+    const int et = ew * 32 + lane;
+    const uint32_t lane_addr = static_cast<uint32_t>(q * 32) << 16;
+    const int c0 = quarter * EPI_COLS;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    float pf_scale = 0.f, pf_inv = 0.f;
+    auto prefetch = [&](const Item& nx) {
+      const int j = nx.col0 + et;
+      pf_scale = (et < TILE && j < nx.n) ? __ldg(ws.inv_norm + nx.base + j) : __int_as_float(0x7fc00000);
+      const int r = nx.row0 + HALF * static_cast<int>(rank) + q * 32 + lane;
+      const bool col = (nx.col0 + c0) / HALF > (nx.row0 + HALF * static_cast<int>(rank)) / HALF;
+      pf_inv = (col && r < nx.n) ? __ldg(ws.inv_norm + nx.base + r) : 0.f;
+    };
+    const uint32_t empty_leader0 = map_to_rank(ptx::smem_addr(&ctl->acc_empty[0]), 0);
+    const uint32_t empty_leader1 = map_to_rank(ptx::smem_addr(&ctl->acc_empty[1]), 0);
+    if (count > 0) prefetch(item(0));
+    for (int64_t k = 0; k < count; ++k) {
+      const Item it = item(k);
+      float* sc = scale + acc * TILE;
+      if (et < TILE) sc[et] = pf_scale;  // NaN outside the image: never wins
+      const float inv_i = pf_inv;
+      ptx::mbar_arrive(&ctl->scale_ready[acc]);
+      if (!ptx::mbar_wait(&ctl->scale_ready[acc], acc_phase, abort_flag, WAIT_LIMIT_NS) ||
+          !ptx::mbar_wait(&ctl->acc_full[acc], acc_phase, abort_flag, WAIT_LIMIT_NS)) {
+        fail(ctl, ws.status, 14);
+        break;
+      }
+      if (k + 1 < count) prefetch(item(k + 1));
+      ptx::tc_fence_after_sync();
+      const int row_base = it.row0 + HALF * static_cast<int>(rank) + q * 32;
+      const int row = row_base + lane;
+      const int jd = row - it.col0;
+      const int iblk = (it.row0 + HALF * static_cast<int>(rank)) / HALF;
+      const int jblk = (it.col0 + c0) / HALF;
+      const bool diag = jblk == iblk;
+      const bool read = jblk >= iblk;
+      const bool col_update = jblk > iblk;
+      float best = -INFINITY;
+      int bj = -1;
+      if (read) {
+#pragma unroll 1
+        for (int c = c0; c < c0 + EPI_COLS; c += 32) {
+          uint32_t v[32];
+          ptx::tmem_ld_32x32b_x32(tmem + lane_addr + static_cast<uint32_t>(acc * TILE + c), v);
+          ptx::tmem_wait_ld(v);
+          unsigned long long* ck = ctl->colkey[acc];
+          if (diag) {
+            chunk<true, false>(v, sc, c, jd, best, bj, inv_i, lane, row_base, it.n, it.col0, ck);
+          } else if (col_update) {
+            chunk<false, true>(v, sc, c, jd, best, bj, inv_i, lane, row_base, it.n, it.col0, ck);
+          }
+        }
+      }
+      ptx::tc_fence_before_sync();
+      if (leader) {
+        ptx::mbar_arrive(&ctl->acc_empty[acc]);
+      } else {
+        __syncwarp();
+        if (lane == 0) remote_arrive(acc == 0 ? empty_leader0 : empty_leader1);
+      }
+      if (bj >= 0 && row < it.n) atomicMax(ws.keys + it.base + row, make_key(best, it.col0 + bj));
+      __threadfence_block();
+      __syncwarp();
+      int last = 0;
+      if (lane == 0) last = atomicAdd(&ctl->colcount[acc], 1) == EPI_WARPS - 1;
+      last = __shfl_sync(0xFFFFFFFFu, last, 0);
+      if (last) {
+        __threadfence_block();
+        for (int e = lane; e < TILE; e += 32) {
+          const unsigned long long key = ctl->colkey[acc][e];
+          if (key != 0ull) {
+            atomicMax(ws.keys + it.base + it.col0 + e, key);
+            ctl->colkey[acc][e] = 0ull;
+          }
+        }
+        if (lane == 0) ctl->colcount[acc] = 0;
+        __threadfence_block();
+      }
+      if (++acc == 2) {
+        acc = 0;
+        acc_phase ^= 1u;
+      }
+    }
+  }
+
+  ptx::tc_fence_before_sync();
+  __syncthreads();
+  cluster_sync();  // no CTA leaves while its peer may still signal it
+  if (warp == 1) {
+    ptx::tc_fence_after_sync();
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TMEM_COLS) : "memory");
+  }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      return static_cast<PFN_cuTensorMapEncodeTiled_v12000>(nullptr);
+    return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }();
+  return fn;
+}
+
+}  // namespace
+
+AffinityTile pair_tile() { return {TILE, TILE, AffinityTile::kUpperSquare}; }
+
+cudaError_t launch_affinity_pair(const void* tokens, int batch, int64_t rows, int dim, const Workspace& ws,
+                                 int num_sms, cudaStream_t stream) {
+  PFN_cuTensorMapEncodeTiled_v12000 encode = encoder();
+  if (encode == nullptr) return cudaErrorNotSupported;
+  CUtensorMap map;
+  const cuuint64_t gdim[2] = {static_cast<cuuint64_t>(dim), static_cast<cuuint64_t>(rows)};
+  const cuuint64_t gstride[1] = {static_cast<cuuint64_t>(dim) * 2};
+  const cuuint32_t box[2] = {BK, HALF};
+  const cuuint32_t estride[2] = {1, 1};
+  if (encode(&map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(tokens), gdim, gstride, box, estride,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return cudaErrorInvalidValue;
+  static std::atomic<uint64_t> attr_done{0};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const uint64_t bit = 1ull << (dev & 63);
+  if (!(attr_done.load() & bit)) {
+    e = cudaFuncSetAttribute(affinity_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(SMEM_BYTES));
+    if (e != cudaSuccess) return e;
+    attr_done.fetch_or(bit);
+  }
+  const int ksteps = (dim + BK - 1) / BK;
+  const int grid = (num_sms > 1 ? num_sms : 2) & ~1;  // whole SM pairs
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(THREADS);
+  cfg.dynamicSmemBytes = SMEM_BYTES;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, affinity_pair_kernel, map, batch, ksteps, ws);
+}
+
+}  // namespace mpm

@@ -101,7 +101,7 @@ __global__ void __launch_bounds__(kThreads) affinity_simt_kernel(const uint8_t* 
 
 }  // namespace
 
-AffinityTile simt_tile() { return {BM, BN, false}; }
+AffinityTile simt_tile() { return {BM, BN, AffinityTile::kDense}; }
 
 cudaError_t launch_affinity_simt(const void* tokens, int batch, int dim, bool bf16, const Workspace& ws,
                                  int num_sms, cudaStream_t stream) {

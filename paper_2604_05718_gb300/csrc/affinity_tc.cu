@@ -79,9 +79,6 @@ struct Control {
   int abort_flag;
 };
 
-constexpr size_t SMEM_BYTES = 1024 + static_cast<size_t>(STAGES) * STAGE_BYTES + 2 * BN * sizeof(float) +
-                              sizeof(Control);
-
 struct Item {
   int64_t base;  // first row of the image
   int n;         // tokens in the image
@@ -90,6 +87,14 @@ struct Item {
   bool upper_only;  // symmetric mode: block 2T lies below the diagonal, so only
                     // block 2T+1 (the diagonal block) is loaded and multiplied
 };
+
+// A CTA decodes its first kMaxItems work items once, at kernel start, into
+// shared memory (one binary search per item, done in parallel) instead of
+// every role repeating the search for every tile.
+constexpr int kMaxItems = 160;
+
+constexpr size_t SMEM_BYTES = 1024 + static_cast<size_t>(STAGES) * STAGE_BYTES + 2 * BN * sizeof(float) +
+                              sizeof(Control) + 16 + kMaxItems * sizeof(Item);
 
 template <bool SYM>
 __device__ __forceinline__ Item decode_item(const Workspace& ws, int batch, int64_t w) {
@@ -196,8 +201,18 @@ __global__ void __launch_bounds__(THREADS, 1)
   uint8_t* stages = smem;
   float* scale = reinterpret_cast<float*>(smem + STAGES * STAGE_BYTES);  // [2][BN]
   Control* ctl = reinterpret_cast<Control*>(smem + STAGES * STAGE_BYTES + 2 * BN * sizeof(float));
+  Item* items = reinterpret_cast<Item*>(
+      (reinterpret_cast<uintptr_t>(ctl + 1) + 15) & ~static_cast<uintptr_t>(15));
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // This CTA's items are w = blockIdx.x + k * gridDim.x, k < count.
+  const int64_t total = __ldg(ws.plan + batch);
+  const int64_t count = total > blockIdx.x ? (total - 1 - blockIdx.x) / gridDim.x + 1 : 0;
+  for (int64_t k = threadIdx.x; k < count && k < kMaxItems; k += THREADS)
+    items[k] = decode_item<SYM>(ws, batch, blockIdx.x + k * gridDim.x);
+  auto item = [&](int64_t k) -> Item {
+    return k < kMaxItems ? items[k] : decode_item<SYM>(ws, batch, blockIdx.x + k * gridDim.x);
+  };
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       ptx::mbar_init(&ctl->full[s], 1);
@@ -225,7 +240,6 @@ __global__ void __launch_bounds__(THREADS, 1)
   __syncthreads();
   ptx::tc_fence_after_sync();
   const uint32_t tmem = ctl->tmem_base;
-  const int64_t total = __ldg(ws.plan + batch);
   volatile int* abort_flag = &ctl->abort_flag;
 
   if (warp == 0) {
@@ -236,8 +250,8 @@ __global__ void __launch_bounds__(THREADS, 1)
       int issued = 0;                 // bit s: stage s has a load in flight or landed
       uint32_t issued_phase = 0;      // bit s: parity of that load's phase
       bool ok = true;
-      for (int64_t w = blockIdx.x; ok && w < total; w += gridDim.x) {
-        const Item it = decode_item<SYM>(ws, batch, w);
+      for (int64_t k = 0; ok && k < count; ++k) {
+        const Item it = item(k);
         const int32_t arow = static_cast<int32_t>(it.base + it.row0);
         const int32_t brow = static_cast<int32_t>(it.base + it.col0);
         for (int kb = 0; kb < ksteps; ++kb) {
@@ -273,10 +287,10 @@ __global__ void __launch_bounds__(THREADS, 1)
       int stage = 0, acc = 0;
       uint32_t phase = 0, acc_phase = 0;
       bool ok = true;
-      for (int64_t w = blockIdx.x; ok && w < total; w += gridDim.x) {
+      for (int64_t k = 0; ok && k < count; ++k) {
         // Tiles whose lower 128-column block is below the diagonal multiply
         // only the upper block (N = 128) into the upper half of the accumulator.
-        const bool upper_only = SYM && decode_item<SYM>(ws, batch, w).upper_only;
+        const bool upper_only = SYM && item(k).upper_only;
         const uint32_t idesc = upper_only ? IDESC_HALF : IDESC;
         const uint32_t b_off = upper_only ? B_BYTES / 2 : 0;
         if (!ptx::mbar_wait(&ctl->acc_empty[acc], acc_phase ^ 1u, abort_flag, WAIT_LIMIT_NS)) {
@@ -328,19 +342,30 @@ __global__ void __launch_bounds__(THREADS, 1)
     const uint32_t lane_addr = static_cast<uint32_t>(q * 32) << 16;
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int64_t w = blockIdx.x; w < total; w += gridDim.x) {
-      const Item it = decode_item<SYM>(ws, batch, w);
+    // The global values a tile needs (its column scale for this thread, and
+    // 1/|x_i| of this thread's row when it takes column candidates) are
+    // fetched one tile ahead, so their latency hides behind the current tile.
+    float pf_scale = 0.f, pf_inv = 0.f;
+    auto prefetch = [&](const Item& nx) {
+      const int j = nx.col0 + et;
+      pf_scale = (et < BN && j < nx.n) ? __ldg(ws.inv_norm + nx.base + j) : __int_as_float(0x7fc00000);
+      const int r = nx.row0 + q * 32 + lane;
+      const bool col = SYM && (nx.col0 + quarter * EPI_COLS) / BM > nx.row0 / BM;
+      pf_inv = (col && r < nx.n) ? __ldg(ws.inv_norm + nx.base + r) : 0.f;
+    };
+    if (count > 0) prefetch(item(0));
+    for (int64_t k = 0; k < count; ++k) {
+      const Item it = item(k);
       float* sc = scale + acc * BN;
-      if (et < BN) {
-        const int j = it.col0 + et;
-        sc[et] = j < it.n ? __ldg(ws.inv_norm + it.base + j) : __int_as_float(0x7fc00000);  // NaN never wins
-      }
+      if (et < BN) sc[et] = pf_scale;  // NaN for columns outside the image: never wins
+      const float inv_i = pf_inv;
       ptx::mbar_arrive(&ctl->scale_ready[acc]);
       if (!ptx::mbar_wait(&ctl->scale_ready[acc], acc_phase, abort_flag, WAIT_LIMIT_NS) ||
           !ptx::mbar_wait(&ctl->acc_full[acc], acc_phase, abort_flag, WAIT_LIMIT_NS)) {
         fail(ctl, ws.status, 4);
         break;
       }
+      if (k + 1 < count) prefetch(item(k + 1));
       ptx::tc_fence_after_sync();
       const int row_base = it.row0 + q * 32;
       const int row = row_base + lane;             // local row owned by this thread
@@ -353,7 +378,6 @@ __global__ void __launch_bounds__(THREADS, 1)
       const bool diag = jblk == iblk;
       const bool read = !SYM || jblk >= iblk;
       const bool col_update = SYM && jblk > iblk;
-      const float inv_i = (col_update && row < it.n) ? __ldg(ws.inv_norm + it.base + row) : 0.f;
       float best = -INFINITY;
       int bj = -1;
       if (read) {
@@ -444,7 +468,9 @@ cudaError_t ensure_smem_attr() {
 
 }  // namespace
 
-AffinityTile tc_tile(bool symmetric) { return {BM, BN, symmetric}; }
+AffinityTile tc_tile(bool symmetric) {
+  return {BM, BN, symmetric ? AffinityTile::kSymmetric : AffinityTile::kDense};
+}
 
 bool tc_available() { return get_encode() != nullptr; }
 

@@ -16,6 +16,9 @@ namespace mpm {
 // grid can be set up while the previous kernel in the stream drains, and
 // starts by waiting for that kernel's completion and memory flush.
 __device__ __forceinline__ void wait_for_previous_grid() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+// Lets the next kernel in the stream be scheduled onto SMs this grid frees;
+// it still waits (wait_for_previous_grid) for this grid to finish.
+__device__ __forceinline__ void allow_next_grid() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
 template <typename... Params, typename... Args>
 inline cudaError_t launch_dependent(void (*kernel)(Params...), dim3 grid, dim3 block, size_t smem,
@@ -63,9 +66,11 @@ __device__ __forceinline__ int find_item_image(const int64_t* __restrict__ plan,
 // every rows x cols tile.  Symmetric (cols == 2 * rows): row block I needs
 // only the column tiles T holding a block J >= I, i.e. 2T + 1 >= I, so it
 // has C - (I >> 1) of them; row blocks 2m and 2m+1 have 2(C - m) together.
-__host__ __device__ __forceinline__ int64_t affinity_tiles(int64_t n, int rows, int cols, bool symmetric) {
+// Upper square (rows == cols): the R (R + 1) / 2 tiles with J >= I.
+__host__ __device__ __forceinline__ int64_t affinity_tiles(int64_t n, int rows, int cols, int mode) {
   const int64_t r = (n + rows - 1) / rows, c = (n + cols - 1) / cols;
-  if (!symmetric) return r * c;
+  if (mode == AffinityTile::kDense) return r * c;
+  if (mode == AffinityTile::kUpperSquare) return r * (r + 1) / 2;
   const int64_t q = r / 2;
   return 2 * q * c - q * (q - 1) + (r & 1) * (c - q);
 }

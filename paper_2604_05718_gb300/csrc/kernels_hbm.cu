@@ -42,6 +42,11 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(const uint8_t* __restric
                                                         bool bf16, AffinityTile tile,
                                                         Workspace ws) {
   wait_for_previous_grid();
+  // The affinity kernel that follows only sets up barriers and tensor memory
+  // before it waits for this grid, so it may take SMs as this grid drains.
+  // (The other kernels do not trigger early: blocks of a dependent grid
+  // parked on SMs were measured to slow the bandwidth-bound kernels.)
+  allow_next_grid();
   if (blockIdx.x == 0) {
     __shared__ int64_t sh[32];
     __shared__ int bad;
@@ -80,7 +85,7 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(const uint8_t* __restric
       int64_t items = 0;
       if (idx < batch) {
         const int64_t n = ws.soff[idx + 1] - ws.soff[idx];
-        items = affinity_tiles(n, tile.rows, tile.cols, tile.symmetric);
+        items = affinity_tiles(n, tile.rows, tile.cols, tile.mode);
       }
       int64_t total;
       const int64_t incl = block_incl_sum<int64_t>(items, sh, &total);

@@ -22,13 +22,17 @@ struct Workspace {
   int2* reps;                 // int2[rows] (representative, partner or -1), per image
 };
 
-// Tile of one affinity work item: rows x columns of the cosine matrix.
-// symmetric: only tiles holding a 128-block at or above the diagonal are
-// computed (requires cols == 2 * rows).
+// Tile of one affinity work item: rows x columns of the cosine matrix, and
+// which tiles of an image's N x N matrix are computed:
+//   kDense        all of them;
+//   kSymmetric    those holding a rows-block at or above the diagonal
+//                 (cols == 2 * rows);
+//   kUpperSquare  the square tiles on or above the diagonal (rows == cols).
 struct AffinityTile {
+  enum Mode : int { kDense = 0, kSymmetric = 1, kUpperSquare = 2 };
   int rows;
   int cols;
-  bool symmetric;
+  int mode;
 };
 
 // Inverse row norms, key reset, offsets sanitisation and the work plan.
@@ -46,6 +50,11 @@ cudaError_t launch_affinity_tc(const void* tokens, int batch, int64_t rows, int 
                                const Workspace& ws, int num_sms, cudaStream_t stream);
 AffinityTile tc_tile(bool symmetric);
 bool tc_available();
+
+// Symmetric affinity + arg max on SM pairs (tcgen05.mma.cta_group::2, bf16).
+cudaError_t launch_affinity_pair(const void* tokens, int batch, int64_t rows, int dim, const Workspace& ws,
+                                 int num_sms, cudaStream_t stream);
+AffinityTile pair_tile();
 
 // Mutual check, representative scan, per-image counts, output offsets.
 cudaError_t launch_mutual_compact(int batch, const Workspace& ws, int32_t* out_map,

@@ -97,30 +97,41 @@ mpm_status check_tokens(const void* tokens, int64_t rows, int32_t dim, mpm_dtype
 
 // Kernel used when the caller does not choose one: the symmetric tensor-core
 // kernel for bf16, CUDA-core fp32 FMA for fp32 (faithful to fp32 inputs).
-mpm_nn_algo default_algo(mpm_dtype dtype) { return dtype == MPM_BF16 ? MPM_NN_TCGEN05_SYM : MPM_NN_SIMT; }
+mpm_nn_algo default_algo(mpm_dtype dtype) { return dtype == MPM_BF16 ? MPM_NN_TCGEN05_PAIR : MPM_NN_SIMT; }
+
+bool is_tensor_core(mpm_nn_algo a) {
+  return a == MPM_NN_TCGEN05 || a == MPM_NN_TCGEN05_SYM || a == MPM_NN_TCGEN05_PAIR;
+}
+
+mpm::AffinityTile tile_of(mpm_nn_algo a) {
+  if (a == MPM_NN_TCGEN05_PAIR) return mpm::pair_tile();
+  if (a == MPM_NN_TCGEN05 || a == MPM_NN_TCGEN05_SYM) return mpm::tc_tile(a == MPM_NN_TCGEN05_SYM);
+  return mpm::simt_tile();
+}
+
+cudaError_t launch_affinity(mpm_nn_algo a, const void* tokens, int batch, int64_t rows, int dim, bool bf16,
+                            const Workspace& ws, int sms, cudaStream_t s) {
+  if (a == MPM_NN_TCGEN05_PAIR) return mpm::launch_affinity_pair(tokens, batch, rows, dim, ws, sms, s);
+  if (a == MPM_NN_TCGEN05 || a == MPM_NN_TCGEN05_SYM)
+    return mpm::launch_affinity_tc(tokens, batch, rows, dim, a == MPM_NN_TCGEN05_SYM, ws, sms, s);
+  return mpm::launch_affinity_simt(tokens, batch, dim, bf16, ws, sms, s);
+}
 
 // The affinity + arg max stage shared by mpm_merge and mpm_nearest_neighbors.
 mpm_status run_affinity(const void* tokens, const int64_t* offsets, int32_t batch, int64_t rows, int32_t dim,
                         mpm_dtype dtype, mpm_nn_algo algo, const Workspace& ws, cudaStream_t stream) {
   const bool bf16 = dtype == MPM_BF16;
   if (algo == MPM_NN_AUTO) algo = default_algo(dtype);
-  const bool tc = algo == MPM_NN_TCGEN05 || algo == MPM_NN_TCGEN05_SYM;
+  const bool tc = is_tensor_core(algo);
   if (algo != MPM_NN_SIMT && !tc) return MPM_ERR_INVALID_ARG;
   if (tc && !bf16) return MPM_ERR_UNSUPPORTED;
   if (tc && !mpm::tc_available()) return MPM_ERR_UNSUPPORTED;
   const int sms = num_sms();
   if (sms <= 0) return MPM_ERR_CUDA;
-  const bool sym = algo == MPM_NN_TCGEN05_SYM;
-  const mpm::AffinityTile tile = tc ? mpm::tc_tile(sym) : mpm::simt_tile();
-  cudaError_t e = mpm::launch_prep(tokens, offsets, batch, rows, dim, bf16, tile, ws, sms, stream);
+  cudaError_t e = mpm::launch_prep(tokens, offsets, batch, rows, dim, bf16, tile_of(algo), ws, sms, stream);
   if (e != cudaSuccess) return MPM_ERR_CUDA;
   if (rows == 0) return MPM_OK;  // every image is empty: nothing to compare
-  if (tc) {
-    e = mpm::launch_affinity_tc(tokens, batch, rows, dim, sym, ws, sms, stream);
-  } else {
-    e = mpm::launch_affinity_simt(tokens, batch, dim, bf16, ws, sms, stream);
-  }
-  return cuda_status(e);
+  return cuda_status(launch_affinity(algo, tokens, batch, rows, dim, bf16, ws, sms, stream));
 }
 
 }  // namespace
@@ -183,8 +194,7 @@ mpm_status mpm_merge_timed(const void* tokens, const int64_t* offsets, int32_t b
   const Workspace ws = carve(workspace, rows, batch);
   const bool bf16 = dtype == MPM_BF16;
   const mpm_nn_algo algo = default_algo(dtype);
-  const bool tc = algo != MPM_NN_SIMT;
-  if (tc && !mpm::tc_available()) return MPM_ERR_UNSUPPORTED;
+  if (is_tensor_core(algo) && !mpm::tc_available()) return MPM_ERR_UNSUPPORTED;
   const int sms = num_sms();
   if (sms <= 0) return MPM_ERR_CUDA;
   // Records stage_events[idx] (if profiling) on the launch stream.
@@ -192,15 +202,13 @@ mpm_status mpm_merge_timed(const void* tokens, const int64_t* offsets, int32_t b
     if (stage_events == nullptr) return true;
     return cudaEventRecord(static_cast<cudaEvent_t>(stage_events[idx]), s) == cudaSuccess;
   };
-  const bool sym = algo == MPM_NN_TCGEN05_SYM;
-  const mpm::AffinityTile tile = tc ? mpm::tc_tile(sym) : mpm::simt_tile();
+  const mpm::AffinityTile tile = tile_of(algo);
   cudaError_t e = cudaSuccess;
   if (!mark(0)) return MPM_ERR_CUDA;
   e = mpm::launch_prep(tokens, offsets, batch, rows, dim, bf16, tile, ws, sms, s);
   if (e != cudaSuccess || !mark(1) || !mark(2)) return MPM_ERR_CUDA;
   if (rows > 0) {
-    e = tc ? mpm::launch_affinity_tc(tokens, batch, rows, dim, sym, ws, sms, s)
-           : mpm::launch_affinity_simt(tokens, batch, dim, bf16, ws, sms, s);
+    e = launch_affinity(algo, tokens, batch, rows, dim, bf16, ws, sms, s);
     if (e != cudaSuccess) return MPM_ERR_CUDA;
   }
   if (!mark(3) || !mark(4)) return MPM_ERR_CUDA;

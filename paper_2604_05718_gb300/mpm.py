@@ -20,7 +20,7 @@ import torch
 LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libmpm.so")
 
 MPM_F32, MPM_BF16 = 0, 1
-ALGOS = {"auto": 0, "simt": 1, "tcgen05": 2, "tcgen05_sym": 3}
+ALGOS = {"auto": 0, "simt": 1, "tcgen05": 2, "tcgen05_sym": 3, "tcgen05_pair": 4}
 STATUS_NAMES = {
     0: "MPM_OK", 1: "MPM_ERR_INVALID_ARG", 2: "MPM_ERR_UNSUPPORTED", 3: "MPM_ERR_ALIGNMENT",
     4: "MPM_ERR_WORKSPACE", 5: "MPM_ERR_CUDA", 6: "MPM_ERR_DEVICE_CHECK", 7: "MPM_ERR_DEVICE_TIMEOUT",

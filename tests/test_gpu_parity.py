@@ -60,7 +60,7 @@ def merge_parity(mpm, batch, what: str, algo: str = "auto") -> ParityStats:
 RAGGED = [0, 1, 2, 3, 127, 128, 129, 255, 256, 257, 300, 1000]
 
 
-@pytest.mark.parametrize("algo", ["tcgen05_sym", "tcgen05"])
+@pytest.mark.parametrize("algo", ["tcgen05_pair", "tcgen05_sym", "tcgen05"])
 @pytest.mark.parametrize("dim", [8, 64, 200, 384, 1024])
 def test_bf16_ragged_tcgen05(mpm, dim, algo):
     batch = make_custom(RAGGED, dim, "bf16", seed=dim)
@@ -83,8 +83,8 @@ def test_f32_ragged(mpm, dim):
     merge_parity(mpm, batch, f"f32 d={dim}")
 
 
-@pytest.mark.parametrize("dtype,algo", [("bf16", "auto"), ("bf16", "tcgen05"), ("bf16", "simt"),
-                                        ("f32", "auto"), ("f32", "simt")])
+@pytest.mark.parametrize("dtype,algo", [("bf16", "auto"), ("bf16", "tcgen05_sym"), ("bf16", "tcgen05"),
+                                        ("bf16", "simt"), ("f32", "auto"), ("f32", "simt")])
 def test_hand_examples_on_gpu(mpm, dtype, algo):
     """Every hand-worked example, packed into one ragged batch, zero-padded to 64 features."""
     exs = load_hand_examples()
@@ -105,8 +105,8 @@ def test_hand_examples_on_gpu(mpm, dtype, algo):
         np.testing.assert_array_equal(g["out"][o0:o1], want, err_msg=e.name)
 
 
-@pytest.mark.parametrize("dtype,algo", [("bf16", "tcgen05_sym"), ("bf16", "tcgen05"), ("bf16", "simt"),
-                                        ("f32", "simt")])
+@pytest.mark.parametrize("dtype,algo", [("bf16", "tcgen05_pair"), ("bf16", "tcgen05_sym"), ("bf16", "tcgen05"),
+                                        ("bf16", "simt"), ("f32", "simt")])
 def test_exact_ties_duplicates_and_zero_rows(mpm, dtype, algo):
     rng = np.random.default_rng(5)
     dim = 64
@@ -132,7 +132,7 @@ def test_exact_ties_duplicates_and_zero_rows(mpm, dtype, algo):
     check_merge_batch(xs, offsets, g["nn"], g["map"], g["out"], g["out_offsets"], dtype, "ties")
 
 
-@pytest.mark.parametrize("algo", ["tcgen05_sym", "tcgen05"])
+@pytest.mark.parametrize("algo", ["tcgen05_pair", "tcgen05_sym", "tcgen05"])
 def test_large_dim_and_large_image(mpm, algo):
     batch = make_custom([300, 77], 4096, "bf16", seed=41)
     merge_parity(mpm, batch, "d=4096", algo=algo)
@@ -142,18 +142,20 @@ def test_large_dim_and_large_image(mpm, algo):
 
 def test_tcgen05_and_simt_agree(mpm):
     batch = make_custom([1000, 513, 64, 2300], 384, "bf16", seed=9)
-    runs = {algo: run_merge(mpm, batch.tokens, batch.offsets, algo) for algo in ("tcgen05", "tcgen05_sym", "simt")}
+    runs = {algo: run_merge(mpm, batch.tokens, batch.offsets, algo)
+            for algo in ("tcgen05", "tcgen05_sym", "tcgen05_pair", "simt")}
     res = [oracle.merge_image(batch.tokens[batch.offsets[k]:batch.offsets[k + 1]].double().numpy())
            for k in range(batch.batch)]
     decisive = np.concatenate([~r.nn.near_tie for r in res])
-    for algo in ("tcgen05_sym", "simt"):
+    for algo in ("tcgen05_sym", "tcgen05_pair", "simt"):
         assert np.array_equal(runs["tcgen05"]["nn"][decisive], runs[algo]["nn"][decisive]), algo
         np.testing.assert_allclose(runs["tcgen05"]["score"], runs[algo]["score"], rtol=0, atol=1e-5)
-    # Dense and symmetric tilings see the very same dot products: identical results.
+    # Every tensor-core tiling sees the very same dot products: identical results.
     assert np.array_equal(runs["tcgen05"]["nn"], runs["tcgen05_sym"]["nn"])
+    assert np.array_equal(runs["tcgen05"]["nn"], runs["tcgen05_pair"]["nn"])
 
 
-@pytest.mark.parametrize("algo", ["tcgen05_sym", "tcgen05"])
+@pytest.mark.parametrize("algo", ["tcgen05_pair", "tcgen05_sym", "tcgen05"])
 def test_scores_are_cosines(mpm, algo):
     batch = make_custom([500, 300], 256, "bf16", seed=3)
     g = run_merge(mpm, batch.tokens, batch.offsets, algo)
