@@ -33,6 +33,7 @@
 #include <atomic>
 
 #include "mpm.h"
+#include "affinity_epilogue.cuh"
 #include "common.cuh"
 #include "ptx.cuh"
 
@@ -59,10 +60,7 @@ struct Control {
   uint64_t empty[STAGES];       // both: MMAs reading stage s completed
   uint64_t acc_full[2];         // both: accumulator a complete
   uint64_t acc_empty[2];        // leader: both CTAs finished reading accumulator a
-  uint64_t scale_ready[2];      // local: column scales of accumulator a written
   uint64_t drain;               // leader: all MMAs completed
-  unsigned long long colkey[2][TILE];
-  int colcount[2];
   uint32_t tmem_base;
   int abort_flag;
 };
@@ -74,9 +72,9 @@ struct Item {
   int col0;  // first local column of the tile (a multiple of 256)
 };
 
-constexpr size_t SMEM_BYTES = 1024 + static_cast<size_t>(STAGES) * STAGE_BYTES + 2 * TILE * sizeof(float) +
+constexpr size_t SMEM_BYTES = 1024 + static_cast<size_t>(STAGES) * STAGE_BYTES + EPI_WARPS * EPI_COLS * sizeof(float) +
                               sizeof(Control) + 16 + kMaxItems * sizeof(Item) +
-                              2 * (kMaxStagedImages + 1) * sizeof(int64_t);
+                              2 * (kMaxStagedImages + 1) * sizeof(int64_t) + EPI_WARPS * 32 * sizeof(uint2);
 
 // Item w of the launch: image by the plan, then the upper-triangle tile (I, J),
 // J >= I, numbered row by row: row I starts at P(I) = I R - I (I - 1) / 2.
@@ -129,8 +127,12 @@ __device__ __forceinline__ uint32_t map_to_rank(uint32_t saddr, uint32_t rank) {
 __device__ __forceinline__ void cluster_sync() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
+// Arrive on an mbarrier of the peer CTA.  The tensor-memory reads this
+// releases are ordered by tcgen05.fence::before_thread_sync, so the arrive
+// itself keeps the default (CTA-scope) semantics and does not wait for this
+// thread's outstanding global atomics.
 __device__ __forceinline__ void remote_arrive(uint32_t cluster_addr) {
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+  asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
 }
 // TMA tile load into this CTA's shared memory whose completion is counted on
 // an mbarrier of either CTA of the pair.
@@ -165,55 +167,9 @@ __device__ __forceinline__ void commit_local(uint64_t* bar) {
                : "memory");
 }
 
-__device__ __forceinline__ int float_order_s32(float x) {
-  const int b = __float_as_int(x);
-  return b ^ ((b >> 31) & 0x7FFFFFFF);
-}
-
 __device__ __forceinline__ void fail(Control* ctl, int32_t* status, int32_t role) {
   ctl->abort_flag = 1;
   report(status, MPM_ERR_DEVICE_TIMEOUT, role);
-}
-
-// One 32-column chunk for the thread's row (see affinity_tc.cu's
-// epilogue_chunk for the reasoning; the arithmetic is the same).
-template <bool DIAG, bool COL>
-__device__ __forceinline__ void chunk(const uint32_t (&v)[32], const float* sc, int c, int jd, float& best, int& bj,
-                                      float inv_i, int lane, int row_base, int n, int col0,
-                                      unsigned long long* colkey) {
-#pragma unroll
-  for (int k = 0; k < 32; k += 4) {
-    const float4 s4 = *reinterpret_cast<const float4*>(sc + c + k);
-    const float sv[4] = {s4.x, s4.y, s4.z, s4.w};
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const float s = __uint_as_float(v[k + u]) * sv[u];
-      if (s > best && (!DIAG || c + k + u != jd)) {
-        best = s;
-        bj = c + k + u;
-      }
-    }
-  }
-  if (COL) {
-    int top = 0;
-    uint32_t lanes = 0;
-#pragma unroll
-    for (int k = 0; k < 32; ++k) {
-      const int key = float_order_s32(__fmaf_rn(__uint_as_float(v[k]), inv_i, 0.0f));
-      const int m = __reduce_max_sync(0xFFFFFFFFu, key);
-      const uint32_t ball = __ballot_sync(0xFFFFFFFFu, key == m);
-      if (lane == k) {
-        top = m;
-        lanes = ball;
-      }
-    }
-    const int winner = row_base + __ffs(static_cast<int>(lanes)) - 1;
-    if (winner < n && col0 + c + lane < n) {
-      const uint32_t hi = static_cast<uint32_t>(top) ^ 0x80000000u;
-      atomicMax(colkey + c + lane, (static_cast<unsigned long long>(hi) << 32) |
-                                       static_cast<unsigned long long>(0xFFFFFFFFu - static_cast<uint32_t>(winner)));
-    }
-  }
 }
 
 __global__ void __launch_bounds__(THREADS, 1)
@@ -221,11 +177,12 @@ __global__ void __launch_bounds__(THREADS, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024u - (ptx::smem_addr(smem_raw) & 1023u)) & 1023u);
   uint8_t* stages = smem;
-  float* scale = reinterpret_cast<float*>(smem + STAGES * STAGE_BYTES);  // [2][TILE]
-  Control* ctl = reinterpret_cast<Control*>(smem + STAGES * STAGE_BYTES + 2 * TILE * sizeof(float));
+  float* scale = reinterpret_cast<float*>(smem + STAGES * STAGE_BYTES);  // [EPI_WARPS][EPI_COLS]
+  Control* ctl = reinterpret_cast<Control*>(smem + STAGES * STAGE_BYTES + EPI_WARPS * EPI_COLS * sizeof(float));
   Item* items = reinterpret_cast<Item*>((reinterpret_cast<uintptr_t>(ctl + 1) + 15) & ~static_cast<uintptr_t>(15));
   int64_t* plan_s = reinterpret_cast<int64_t*>(items + kMaxItems);
   int64_t* soff_s = plan_s + kMaxStagedImages + 1;
+  uint2* scratch_all = reinterpret_cast<uint2*>(soff_s + kMaxStagedImages + 1);  // [EPI_WARPS][32]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = cluster_rank();
@@ -242,15 +199,12 @@ __global__ void __launch_bounds__(THREADS, 1)
       ptx::mbar_init(&ctl->acc_full[a], 1);
       // Leader's threads arrive one by one, the peer's warps once each.
       ptx::mbar_init(&ctl->acc_empty[a], EPI_WARPS * 32 + EPI_WARPS);
-      ptx::mbar_init(&ctl->scale_ready[a], EPI_WARPS * 32);
-      ctl->colcount[a] = 0;
     }
     ptx::mbar_init(&ctl->drain, 1);
     ctl->abort_flag = 0;
     ptx::fence_barrier_init();
     ptx::prefetch_tensor_map(&tmap);
   }
-  for (int e = threadIdx.x; e < 2 * TILE; e += THREADS) (&ctl->colkey[0][0])[e] = 0ull;
   if (warp == 1) {
     // Both CTAs of the pair take part in the joint allocation.
     asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
@@ -370,18 +324,25 @@ __global__ void __launch_bounds__(THREADS, 1)
     __syncwarp();
   } else {
     // ---------------- epilogue (both CTAs) ----------------
+    // Warp (q, quarter) reads tile rows 32q..32q+31 of this CTA and tile
+    // columns c0..c0+63.  It keeps its own copy of those 64 column scales, so
+    // no epilogue warp ever waits for another one.
     const int ew = warp - 2;
     const int q = warp & 3;
     const int quarter = ew >> 2;
-    const int et = ew * 32 + lane;
     const uint32_t lane_addr = static_cast<uint32_t>(q * 32) << 16;
     const int c0 = quarter * EPI_COLS;
+    float* my_scale = scale + ew * EPI_COLS;
+    const float* sc = my_scale - c0;  // indexed by tile column
+    uint2* scr = scratch_all + ew * 32;
     int acc = 0;
     uint32_t acc_phase = 0;
-    float pf_scale = 0.f, pf_inv = 0.f;
+    float pf_scale0 = 0.f, pf_scale1 = 0.f, pf_inv = 0.f;
     auto prefetch = [&](const Item& nx) {
-      const int j = nx.col0 + et;
-      pf_scale = (et < TILE && j < nx.n) ? __ldg(ws.inv_norm + nx.base + j) : __int_as_float(0x7fc00000);
+      const float nan = __int_as_float(0x7fc00000);  // columns outside the image never win
+      const int j0 = nx.col0 + c0 + lane, j1 = j0 + 32;
+      pf_scale0 = j0 < nx.n ? __ldg(ws.inv_norm + nx.base + j0) : nan;
+      pf_scale1 = j1 < nx.n ? __ldg(ws.inv_norm + nx.base + j1) : nan;
       const int r = nx.row0 + HALF * static_cast<int>(rank) + q * 32 + lane;
       const bool col = (nx.col0 + c0) / HALF > (nx.row0 + HALF * static_cast<int>(rank)) / HALF;
       pf_inv = (col && r < nx.n) ? __ldg(ws.inv_norm + nx.base + r) : 0.f;
@@ -391,12 +352,11 @@ __global__ void __launch_bounds__(THREADS, 1)
     if (count > 0) prefetch(item(0));
     for (int64_t k = 0; k < count; ++k) {
       const Item it = item(k);
-      float* sc = scale + acc * TILE;
-      if (et < TILE) sc[et] = pf_scale;  // NaN outside the image: never wins
+      my_scale[lane] = pf_scale0;
+      my_scale[lane + 32] = pf_scale1;
       const float inv_i = pf_inv;
-      ptx::mbar_arrive(&ctl->scale_ready[acc]);
-      if (!ptx::mbar_wait(&ctl->scale_ready[acc], acc_phase, abort_flag, WAIT_LIMIT_NS) ||
-          !ptx::mbar_wait(&ctl->acc_full[acc], acc_phase, abort_flag, WAIT_LIMIT_NS)) {
+      __syncwarp();
+      if (!ptx::mbar_wait(&ctl->acc_full[acc], acc_phase, abort_flag, WAIT_LIMIT_NS)) {
         fail(ctl, ws.status, 14);
         break;
       }
@@ -408,24 +368,21 @@ __global__ void __launch_bounds__(THREADS, 1)
       const int iblk = (it.row0 + HALF * static_cast<int>(rank)) / HALF;
       const int jblk = (it.col0 + c0) / HALF;
       const bool diag = jblk == iblk;
-      const bool read = jblk >= iblk;
       const bool col_update = jblk > iblk;
       float best = -INFINITY;
       int bj = -1;
-      if (read) {
-#pragma unroll 1
-        for (int c = c0; c < c0 + EPI_COLS; c += 32) {
-          uint32_t v[32];
-          ptx::tmem_ld_32x32b_x32(tmem + lane_addr + static_cast<uint32_t>(acc * TILE + c), v);
-          ptx::tmem_wait_ld(v);
-          unsigned long long* ck = ctl->colkey[acc];
-          if (diag) {
-            chunk<true, false>(v, sc, c, jd, best, bj, inv_i, lane, row_base, it.n, it.col0, ck);
-          } else if (col_update) {
-            chunk<false, true>(v, sc, c, jd, best, bj, inv_i, lane, row_base, it.n, it.col0, ck);
-          }
-        }
+      unsigned long long colcand[EPI_COLS / 32];
+#pragma unroll
+      for (int h = 0; h < EPI_COLS / 32; ++h) colcand[h] = 0ull;
+      const uint32_t taddr = tmem + lane_addr + static_cast<uint32_t>(acc * TILE + c0);
+      if (diag) {
+        epilogue_slice<EPI_COLS, true, false>(taddr, sc, c0, jd, best, bj, inv_i, lane, row_base, it.n, it.col0, scr,
+                                              colcand);
+      } else if (col_update) {
+        epilogue_slice<EPI_COLS, false, true>(taddr, sc, c0, jd, best, bj, inv_i, lane, row_base, it.n, it.col0, scr,
+                                              colcand);
       }
+      // Release the accumulator first, then merge this tile's candidates.
       ptx::tc_fence_before_sync();
       if (leader) {
         ptx::mbar_arrive(&ctl->acc_empty[acc]);
@@ -434,23 +391,10 @@ __global__ void __launch_bounds__(THREADS, 1)
         if (lane == 0) remote_arrive(acc == 0 ? empty_leader0 : empty_leader1);
       }
       if (bj >= 0 && row < it.n) atomicMax(ws.keys + it.base + row, make_key(best, it.col0 + bj));
-      __threadfence_block();
-      __syncwarp();
-      int last = 0;
-      if (lane == 0) last = atomicAdd(&ctl->colcount[acc], 1) == EPI_WARPS - 1;
-      last = __shfl_sync(0xFFFFFFFFu, last, 0);
-      if (last) {
-        __threadfence_block();
-        for (int e = lane; e < TILE; e += 32) {
-          const unsigned long long key = ctl->colkey[acc][e];
-          if (key != 0ull) {
-            atomicMax(ws.keys + it.base + it.col0 + e, key);
-            ctl->colkey[acc][e] = 0ull;
-          }
-        }
-        if (lane == 0) ctl->colcount[acc] = 0;
-        __threadfence_block();
-      }
+#pragma unroll
+      for (int h = 0; h < EPI_COLS / 32; ++h)
+        if (colcand[h] != 0ull) atomicMax(ws.keys + it.base + it.col0 + c0 + 32 * h + lane, colcand[h]);
+      __syncwarp();  // all lanes done reading my_scale before the next tile overwrites it
       if (++acc == 2) {
         acc = 0;
         acc_phase ^= 1u;

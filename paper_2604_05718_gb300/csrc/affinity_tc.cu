@@ -44,6 +44,7 @@
 #include <mutex>
 
 #include "mpm.h"
+#include "affinity_epilogue.cuh"
 #include "common.cuh"
 #include "ptx.cuh"
 
@@ -94,7 +95,7 @@ struct Item {
 constexpr int kMaxItems = 160;
 
 constexpr size_t SMEM_BYTES = 1024 + static_cast<size_t>(STAGES) * STAGE_BYTES + 2 * BN * sizeof(float) +
-                              sizeof(Control) + 16 + kMaxItems * sizeof(Item);
+                              sizeof(Control) + 16 + kMaxItems * sizeof(Item) + EPI_WARPS * 32 * sizeof(uint2);
 
 template <bool SYM>
 __device__ __forceinline__ Item decode_item(const Workspace& ws, int batch, int64_t w) {
@@ -134,64 +135,6 @@ __device__ __forceinline__ void fail(Control* ctl, int32_t* status, int32_t role
   report(status, MPM_ERR_DEVICE_TIMEOUT, role);
 }
 
-// Signed-integer order of fp32 values: a < b as floats iff f(a) < f(b) as
-// int32 (negative floats have their magnitude bits flipped).  f(x) with the
-// sign bit flipped equals order_f32(x).  -0 sorts below +0, so scores are
-// canonicalised first.
-__device__ __forceinline__ int float_order_s32(float x) {
-  const int b = __float_as_int(x);
-  return b ^ ((b >> 31) & 0x7FFFFFFF);
-}
-
-// One 32-column chunk of the epilogue for the thread's row: row candidates
-// (best column by G_ij / |x_j|), skipping the diagonal when DIAG, and, when
-// COL, the column candidates (best row of the warp by G_ij / |x_i|).
-template <bool DIAG, bool COL>
-__device__ __forceinline__ void epilogue_chunk(const uint32_t (&v)[32], const float* sc, int c, int jd,
-                                               float& best, int& bj, float inv_i, int lane, int row_base,
-                                               int n, int col0, unsigned long long* colkey) {
-#pragma unroll
-  for (int k = 0; k < 32; k += 4) {
-    const float4 s4 = *reinterpret_cast<const float4*>(sc + c + k);
-    const float sv[4] = {s4.x, s4.y, s4.z, s4.w};
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const float s = __uint_as_float(v[k + u]) * sv[u];
-      if (s > best && (!DIAG || c + k + u != jd)) {
-        best = s;
-        bj = c + k + u;
-      }
-    }
-  }
-  if (COL) {
-    // Column j = col0 + c + k scores this row by G_ij / |x_i|.  fma(v, inv, +0)
-    // is the rounded product with -0 folded into +0, so equal scores order
-    // equally.  Per column: the warp's best ordered score (one warp max) and
-    // the lanes holding it (one ballot); lane k keeps column k's result.
-    // Rows outside the image only occur in an image's last row block, whose
-    // column updates (blocks J > I) lie wholly outside the image and are
-    // dropped by the column check; the row check below is a second guard.
-    int top = 0;
-    uint32_t lanes = 0;
-#pragma unroll
-    for (int k = 0; k < 32; ++k) {
-      const int key = float_order_s32(__fmaf_rn(__uint_as_float(v[k]), inv_i, 0.0f));
-      const int m = __reduce_max_sync(0xFFFFFFFFu, key);
-      const uint32_t ball = __ballot_sync(0xFFFFFFFFu, key == m);
-      if (lane == k) {
-        top = m;
-        lanes = ball;
-      }
-    }
-    const int winner = row_base + __ffs(static_cast<int>(lanes)) - 1;
-    if (winner < n && col0 + c + lane < n) {
-      const uint32_t hi = static_cast<uint32_t>(top) ^ 0x80000000u;  // = order_f32 of the score
-      atomicMax(colkey + c + lane, (static_cast<unsigned long long>(hi) << 32) |
-                                       static_cast<unsigned long long>(0xFFFFFFFFu - static_cast<uint32_t>(winner)));
-    }
-  }
-}
-
 template <bool SYM>
 __global__ void __launch_bounds__(THREADS, 1)
     affinity_tc_kernel(const __grid_constant__ CUtensorMap tmap, int batch, int ksteps, Workspace ws) {
@@ -203,6 +146,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   Control* ctl = reinterpret_cast<Control*>(smem + STAGES * STAGE_BYTES + 2 * BN * sizeof(float));
   Item* items = reinterpret_cast<Item*>(
       (reinterpret_cast<uintptr_t>(ctl + 1) + 15) & ~static_cast<uintptr_t>(15));
+  uint2* scratch_all = reinterpret_cast<uint2*>(items + kMaxItems);  // [EPI_WARPS][32]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   // This CTA's items are w = blockIdx.x + k * gridDim.x, k < count.
@@ -386,13 +330,15 @@ __global__ void __launch_bounds__(THREADS, 1)
           uint32_t v[32];
           ptx::tmem_ld_32x32b_x32(tmem + lane_addr + static_cast<uint32_t>(acc * BN + c), v);
           ptx::tmem_wait_ld(v);
-          unsigned long long* ck = ctl->colkey[acc];
+          uint2* scr = scratch_all + ew * 32;
           if (diag) {
-            epilogue_chunk<true, false>(v, sc, c, jd, best, bj, inv_i, lane, row_base, it.n, it.col0, ck);
+            epilogue_chunk<true, false>(v, sc, c, jd, best, bj, inv_i, lane, row_base, it.n, it.col0, scr);
           } else if (col_update) {
-            epilogue_chunk<false, true>(v, sc, c, jd, best, bj, inv_i, lane, row_base, it.n, it.col0, ck);
+            const unsigned long long key =
+                epilogue_chunk<false, true>(v, sc, c, jd, best, bj, inv_i, lane, row_base, it.n, it.col0, scr);
+            if (key != 0ull) atomicMax(&ctl->colkey[acc][c + lane], key);
           } else {
-            epilogue_chunk<false, false>(v, sc, c, jd, best, bj, inv_i, lane, row_base, it.n, it.col0, ck);
+            epilogue_chunk<false, false>(v, sc, c, jd, best, bj, inv_i, lane, row_base, it.n, it.col0, scr);
           }
         }
       }
