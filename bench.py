@@ -44,7 +44,8 @@ PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 L2_FLUSH_BYTES = 256 << 20
 KERNELS_PER_MERGE = 4
-TRAFFIC_FILE = os.path.join(ROOT, "profiles", "affinity_tc_traffic.txt")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "affinity_pair_traffic.txt")
+AFFINITY_SOURCE = os.path.join(ROOT, "paper_2604_05718_gb300", "csrc", "affinity_pair.cu")
 
 
 def parse_args():
@@ -468,23 +469,20 @@ def run_mpm(args):
     achieved_tflops = sum(aff_flops) / (sum(aff_ms) * 1e-3) / 1e12
     flops_per_launch = sum(aff_flops) / launches
     tensor_peak = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
-    # What the tensor pipe executes: symmetric 128 x 256 tiles over K padded to 64.
+    # What the tensor pipe executes: the 256 x 256 tiles on or above each
+    # image's diagonal, over K padded to 64.
     kpad = -(-dim // 64) * 64
 
     def exec_flops(ns):
-        tiles = 0
-        for n in ns.astype(np.int64):
-            r, c = -(-n // 128), -(-n // 256)
-            q = r // 2
-            tiles += 2 * q * c - q * (q - 1) + (r & 1) * (c - q)
-        return float(tiles) * 128 * 256 * 2 * kpad
+        r = -(-ns.astype(np.int64) // 256)
+        return float(np.sum(r * (r + 1) // 2)) * 256 * 256 * 2 * kpad
 
     exe = [exec_flops(n0)] * args.steps + ([exec_flops(n1)] * args.steps if two else [])
     executed_tflops = sum(exe) / (sum(aff_ms) * 1e-3) / 1e12
     rows_per_launch = (n0.sum() + (n1.sum() if two else 0.0)) / (2.0 if two else 1.0)
-    traffic = traffic_for(os.path.join(ROOT, "paper_2604_05718_gb300", "csrc", "affinity_tc.cu"), rows_per_launch)
+    traffic = traffic_for(AFFINITY_SOURCE, rows_per_launch)
     roofline = {
-        "kernel": "affinity_tc_kernel<symmetric> (fused cosine affinity + arg max, TMA + tcgen05)",
+        "kernel": "affinity_pair_kernel (fused cosine affinity + arg max, TMA + tcgen05.mma.cta_group::2)",
         "bound": "tensor", "achieved": achieved_tflops, "peak": tensor_peak, "unit": "TFLOP/s",
         "frac": achieved_tflops / tensor_peak,
         "peak_kind": f"{peak_kind} bf16 sustained (kernel timed inside the step loop)",
@@ -493,7 +491,7 @@ def run_mpm(args):
         "frac_of_burst_peak": achieved_tflops / peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]),
         "executed_tflops": executed_tflops,
         "executed_frac": executed_tflops / tensor_peak,
-        "executed_definition": "MMA work issued: symmetric 128x256 tiles x K padded to 64, 2 flops per MAC",
+        "executed_definition": "MMA work issued: 256x256 tiles on or above the diagonal x K padded to 64",
         "traffic": traffic,
     }
     # HBM fractions of the bandwidth kernels (algorithmic bytes / event time).
