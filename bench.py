@@ -470,8 +470,8 @@ def run_mpm(args):
     flops_per_launch = sum(aff_flops) / launches
     tensor_peak = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
     # What the tensor pipe executes: the 256 x 256 tiles on or above each
-    # image's diagonal, over K padded to 64.
-    kpad = -(-dim // 64) * 64
+    # image's diagonal, over K padded to 16 (the MMA's K).
+    kpad = -(-dim // 16) * 16
 
     def exec_flops(ns):
         r = -(-ns.astype(np.int64) // 256)
@@ -491,7 +491,7 @@ def run_mpm(args):
         "frac_of_burst_peak": achieved_tflops / peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]),
         "executed_tflops": executed_tflops,
         "executed_frac": executed_tflops / tensor_peak,
-        "executed_definition": "MMA work issued: 256x256 tiles on or above the diagonal x K padded to 64",
+        "executed_definition": "MMA work issued: 256x256 tiles on or above the diagonal x K padded to 16",
         "traffic": traffic,
     }
     # HBM fractions of the bandwidth kernels (algorithmic bytes / event time).

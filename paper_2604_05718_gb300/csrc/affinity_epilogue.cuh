@@ -68,69 +68,93 @@ __device__ __forceinline__ unsigned long long epilogue_chunk(const uint32_t (&v)
   return 0ull;
 }
 
+// One 16-column piece of a warp's slice: row candidates into two running
+// maxima (even and odd columns), and, with COL, the column maxima and their
+// winning rows of these 16 columns into the per-warp scratch entries
+// slot .. slot + 15.
+template <bool DIAG, bool COL>
+__device__ __forceinline__ void epilogue_piece(const uint32_t (&v)[16], const float* sc, int c, int jd, float& best0,
+                                               int& bj0, float& best1, int& bj1, float inv_i, int lane,
+                                               uint2* scratch, int slot) {
+#pragma unroll
+  for (int k = 0; k < 16; k += 4) {
+    const float4 s4 = *reinterpret_cast<const float4*>(sc + c + k);
+    const float sv[4] = {s4.x, s4.y, s4.z, s4.w};
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const float s = __uint_as_float(v[k + u]) * sv[u];
+      const int j = c + k + u;
+      if (u & 1) {
+        if (s > best1 && (!DIAG || j != jd)) {
+          best1 = s;
+          bj1 = j;
+        }
+      } else {
+        if (s > best0 && (!DIAG || j != jd)) {
+          best0 = s;
+          bj0 = j;
+        }
+      }
+    }
+  }
+  if (COL) {
+    const bool writer = lane == 0;
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+      const float s = __uint_as_float(v[k]) * inv_i;
+      const float m = warp_max_f32(s);
+      const uint32_t ball = __ballot_sync(0xFFFFFFFFu, s == m);
+      if (writer) scratch[slot + k] = make_uint2(__float_as_uint(m), ball);
+    }
+  }
+}
+
+// Column candidate of tile column c + lane from the scratch entries of the
+// 32 columns c .. c + 31 (0 when there is none).
+__device__ __forceinline__ unsigned long long column_candidate(const uint2* scratch, int lane, int row_base, int n,
+                                                               int col) {
+  __syncwarp();
+  const uint2 r = scratch[lane];
+  __syncwarp();
+  const int winner = row_base + __ffs(static_cast<int>(r.y)) - 1;
+  return (r.y != 0u && winner < n && col < n) ? make_key(__uint_as_float(r.x), winner) : 0ull;
+}
+
 // A warp's whole COLS-column slice of one accumulator (TMEM columns
-// tmem_col .. tmem_col + COLS - 1, tile columns c0 ..), read in 16-column
-// pieces with the next piece's load in flight while the current one is
-// processed.  Row candidates use two independent running maxima (even and
-// odd columns), merged at the end with the lowest-index rule, to halve the
-// dependent chain.  colcand[h] receives the column candidate of tile column
+// taddr .. taddr + COLS - 1, tile columns c0 ..), read in 16-column pieces
+// with the next piece's load in flight while the current one is processed.
+// The loop body covers two pieces (32 columns) and is not unrolled further,
+// which keeps the epilogue's code small: the MMA-issuing warp shares its
+// sub-partition's instruction cache with four epilogue warps.  Row
+// candidates use two independent running maxima (even and odd columns),
+// merged at the end with the lowest-index rule, to halve the dependent
+// chain.  colcand[h] receives the column candidate of tile column
 // c0 + 32 h + lane (0 when none).
 template <int COLS, bool DIAG, bool COL>
 __device__ __forceinline__ void epilogue_slice(uint32_t taddr, const float* sc, int c0, int jd, float& best,
                                                int& bj, float inv_i, int lane, int row_base, int n, int col0,
                                                uint2* scratch, unsigned long long (&colcand)[COLS / 32]) {
-  constexpr int PIECES = COLS / 16;
+  static_assert(COLS % 32 == 0, "slices are whole 32-column pairs of pieces");
   float best0 = -INFINITY, best1 = -INFINITY;
   int bj0 = -1, bj1 = -1;
   uint32_t va[16], vb[16];
   ptx::tmem_ld_32x32b_x16(taddr, va);
   ptx::tmem_wait_ld(va);
-#pragma unroll
-  for (int p = 0; p < PIECES; ++p) {
-    uint32_t(&cur)[16] = (p & 1) ? vb : va;
-    uint32_t(&nxt)[16] = (p & 1) ? va : vb;
-    if (p + 1 < PIECES) ptx::tmem_ld_32x32b_x16(taddr + 16 * (p + 1), nxt);
-    const int c = c0 + 16 * p;
-#pragma unroll
-    for (int k = 0; k < 16; k += 4) {
-      const float4 s4 = *reinterpret_cast<const float4*>(sc + c + k);
-      const float sv[4] = {s4.x, s4.y, s4.z, s4.w};
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const float s = __uint_as_float(cur[k + u]) * sv[u];
-        const int j = c + k + u;
-        if (u & 1) {
-          if (s > best1 && (!DIAG || j != jd)) {
-            best1 = s;
-            bj1 = j;
-          }
-        } else {
-          if (s > best0 && (!DIAG || j != jd)) {
-            best0 = s;
-            bj0 = j;
-          }
-        }
-      }
-    }
+#pragma unroll 1
+  for (int h = 0; h < COLS / 32; ++h) {
+    const int c = c0 + 32 * h;
+    ptx::tmem_ld_32x32b_x16(taddr + 32 * h + 16, vb);
+    epilogue_piece<DIAG, COL>(va, sc, c, jd, best0, bj0, best1, bj1, inv_i, lane, scratch, 0);
+    ptx::tmem_wait_ld(vb);
+    if (h + 1 < COLS / 32) ptx::tmem_ld_32x32b_x16(taddr + 32 * h + 32, va);
+    epilogue_piece<DIAG, COL>(vb, sc, c + 16, jd, best0, bj0, best1, bj1, inv_i, lane, scratch, 16);
     if (COL) {
-      const bool writer = lane == 0;
+      const unsigned long long key = column_candidate(scratch, lane, row_base, n, col0 + c + lane);
 #pragma unroll
-      for (int k = 0; k < 16; ++k) {
-        const float s = __uint_as_float(cur[k]) * inv_i;
-        const float m = warp_max_f32(s);
-        const uint32_t ball = __ballot_sync(0xFFFFFFFFu, s == m);
-        if (writer) scratch[16 * (p & 1) + k] = make_uint2(__float_as_uint(m), ball);
-      }
-      if (p & 1) {
-        __syncwarp();
-        const uint2 r = scratch[lane];
-        __syncwarp();
-        const int winner = row_base + __ffs(static_cast<int>(r.y)) - 1;
-        const int cc = c - 16 + lane;  // tile column of this lane's result
-        colcand[p >> 1] = (r.y != 0u && winner < n && col0 + cc < n) ? make_key(__uint_as_float(r.x), winner) : 0ull;
-      }
+      for (int g = 0; g < COLS / 32; ++g)
+        if (g == h) colcand[g] = key;
     }
-    if (p + 1 < PIECES) ptx::tmem_wait_ld(nxt);
+    if (h + 1 < COLS / 32) ptx::tmem_wait_ld(va);
   }
   // Merge the two chains: larger score, lower column on equal scores.
   if (best1 > best0 || (best1 == best0 && bj1 >= 0 && (bj0 < 0 || bj1 < bj0))) {

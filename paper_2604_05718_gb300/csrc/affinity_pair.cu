@@ -10,9 +10,13 @@
 //    G = X X^T with tcgen05.mma.cta_group::2 (M = 256, N = 256).  CTA r holds
 //    tile rows [128r, 128r + 128) of A and tile columns [128r, 128r + 128) of
 //    B in its own shared memory, and receives its 128 rows x 256 columns of
-//    the accumulator in its own tensor memory.  Each SM therefore stages 32
-//    KiB per 64-feature step instead of 48 KiB, which leaves room for six
-//    stages and cuts the shared-memory traffic of the tensor cores by a third.
+//    the accumulator in its own tensor memory.  Each SM therefore stages 64
+//    KiB per 128-feature stage (two 64-feature TMA boxes per operand) instead
+//    of 96 KiB, which leaves room for three stages and cuts the
+//    shared-memory traffic of the tensor cores by a third.  The MMA warp
+//    issues a whole stage (eight MMAs and the release commit) from one asm
+//    block: its sub-partition also runs four epilogue warps, and every
+//    instruction it saves per stage keeps the tensor core fed.
 //  * Tiles are the 256 x 256 blocks on or above the diagonal of each image's
 //    G, R(R + 1) / 2 of them for R = ceil(N_b / 256).  Within a tile, every
 //    128-column block above a thread's 128-row block also yields column
@@ -42,10 +46,13 @@ namespace {
 
 constexpr int TILE = 256;                      // tile rows and columns
 constexpr int HALF = 128;                      // rows of A / B per CTA
-constexpr int BK = 64;
-constexpr int STAGES = 6;
-constexpr int SLICE_BYTES = HALF * BK * 2;     // 16 KiB
-constexpr int STAGE_BYTES = 2 * SLICE_BYTES;   // A slice + B slice of this CTA
+constexpr int BOX_K = 64;                      // features per TMA box: one 128-byte swizzle row
+constexpr int BK = 128;                        // features per pipeline stage
+constexpr int ATOMS = BK / BOX_K;              // swizzle atoms (TMA boxes) per operand slice
+constexpr int ATOM_BYTES = HALF * BOX_K * 2;   // 16 KiB
+constexpr int STAGES = 3;
+constexpr int SLICE_BYTES = ATOMS * ATOM_BYTES;  // 32 KiB: 128 rows x BK features
+constexpr int STAGE_BYTES = 2 * SLICE_BYTES;     // A slice + B slice of this CTA
 constexpr int EPI_WARPS = 16;
 constexpr int EPI_COLS = TILE / (EPI_WARPS / 4);
 constexpr int THREADS = (2 + EPI_WARPS) * 32;
@@ -153,6 +160,42 @@ __device__ __forceinline__ void mma_pair(uint32_t d_tmem, uint64_t a_desc, uint6
       "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
+// The eight K = 16 MMAs of one full stage (BK = 128 features: two swizzle
+// atoms of four 32-byte K slices each), then the commit that releases the
+// stage in both CTAs.  a_desc describes the stage's A slice; the B slice
+// follows it by SLICE_BYTES.  One asm block keeps the issuing thread's
+// instruction stream short: the MMA warp shares its SM sub-partition with
+// four epilogue warps, and the tensor core idles whenever this loop falls
+// behind.
+__device__ __forceinline__ void mma_stage_full(uint32_t d_tmem, uint64_t a_desc, uint32_t idesc, uint32_t accumulate,
+                                               uint64_t* release) {
+  static_assert(ATOMS == 2 && (ATOM_BYTES >> 4) == 1024 && (SLICE_BYTES >> 4) == 2048, "offsets below");
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t.reg .b64 a, b;\n\t"
+      "setp.ne.b32 p, %3, 0;\n\t"
+      "setp.ne.b32 q, %5, 0;\n\t"
+      "add.s64 b, %1, 2048;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, b, %2, p;\n\t"
+      "add.s64 a, %1, 2;\n\tadd.s64 b, %1, 2050;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], a, b, %2, q;\n\t"
+      "add.s64 a, %1, 4;\n\tadd.s64 b, %1, 2052;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], a, b, %2, q;\n\t"
+      "add.s64 a, %1, 6;\n\tadd.s64 b, %1, 2054;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], a, b, %2, q;\n\t"
+      "add.s64 a, %1, 1024;\n\tadd.s64 b, %1, 3072;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], a, b, %2, q;\n\t"
+      "add.s64 a, %1, 1026;\n\tadd.s64 b, %1, 3074;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], a, b, %2, q;\n\t"
+      "add.s64 a, %1, 1028;\n\tadd.s64 b, %1, 3076;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], a, b, %2, q;\n\t"
+      "add.s64 a, %1, 1030;\n\tadd.s64 b, %1, 3078;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], a, b, %2, q;\n\t"
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%4], %6;\n\t}"
+      ::"r"(d_tmem), "l"(a_desc), "r"(idesc), "r"(accumulate), "r"(ptx::smem_addr(release)), "r"(1u),
+      "h"(static_cast<uint16_t>(3))
+      : "memory");
+}
+
 // Arrives on the barrier at this offset in both CTAs once the MMAs issued so
 // far completed.
 __device__ __forceinline__ void commit_both(uint64_t* bar) {
@@ -173,7 +216,7 @@ __device__ __forceinline__ void fail(Control* ctl, int32_t* status, int32_t role
 }
 
 __global__ void __launch_bounds__(THREADS, 1)
-    affinity_pair_kernel(const __grid_constant__ CUtensorMap tmap, int batch, int ksteps, Workspace ws) {
+    affinity_pair_kernel(const __grid_constant__ CUtensorMap tmap, int batch, int dim, Workspace ws) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024u - (ptx::smem_addr(smem_raw) & 1023u)) & 1023u);
   uint8_t* stages = smem;
@@ -187,6 +230,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = cluster_rank();
   const bool leader = rank == 0;
+  const int ksteps = (dim + BK - 1) / BK;
   const int64_t clusters = cluster_count();
   const int64_t cid = cluster_id();
 
@@ -263,8 +307,11 @@ __global__ void __launch_bounds__(THREADS, 1)
           uint8_t* sa = stages + stage * STAGE_BYTES;
           const uint32_t full_leader = map_to_rank(ptx::smem_addr(&ctl->full[stage]), 0);
           if (leader) ptx::mbar_arrive_expect_tx(&ctl->full[stage], 2 * STAGE_BYTES);
-          tma_load_2d_pair(sa, &tmap, full_leader, kb * BK, arow);
-          tma_load_2d_pair(sa + SLICE_BYTES, &tmap, full_leader, kb * BK, brow);
+#pragma unroll
+          for (int t = 0; t < ATOMS; ++t) {
+            tma_load_2d_pair(sa + t * ATOM_BYTES, &tmap, full_leader, kb * BK + t * BOX_K, arow);
+            tma_load_2d_pair(sa + SLICE_BYTES + t * ATOM_BYTES, &tmap, full_leader, kb * BK + t * BOX_K, brow);
+          }
           issued |= 1 << stage;
           issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
           if (++stage == STAGES) {
@@ -285,6 +332,9 @@ __global__ void __launch_bounds__(THREADS, 1)
       int stage = 0, acc = 0;
       uint32_t phase = 0, acc_phase = 0;
       bool ok = true;
+      // Descriptor of stage 0's A slice; the others differ only in the
+      // start-address field (address / 16, no carry out of its 14 bits).
+      const uint64_t desc0 = ptx::sdesc_k_sw128(ptx::smem_addr(stages));
       for (int64_t k = 0; ok && k < count; ++k) {
         if (!ptx::mbar_wait(&ctl->acc_empty[acc], acc_phase ^ 1u, abort_flag, WAIT_LIMIT_NS)) {
           fail(ctl, ws.status, 12);
@@ -299,13 +349,18 @@ __global__ void __launch_bounds__(THREADS, 1)
             break;
           }
           ptx::tc_fence_after_sync();
-          const uint32_t a_addr = ptx::smem_addr(stages + stage * STAGE_BYTES);
-          const uint32_t b_addr = a_addr + SLICE_BYTES;
-#pragma unroll
-          for (int kk = 0; kk < BK / 16; ++kk)
-            mma_pair(d_tmem, ptx::sdesc_k_sw128(a_addr + kk * 32), ptx::sdesc_k_sw128(b_addr + kk * 32), IDESC,
-                     (kb | kk) != 0 ? 1u : 0u);
-          commit_both(&ctl->empty[stage]);
+          const uint64_t a_desc = desc0 + static_cast<uint64_t>((stage * STAGE_BYTES) >> 4);
+          if ((kb + 1) * BK <= dim) {
+            mma_stage_full(d_tmem, a_desc, IDESC, kb != 0 ? 1u : 0u, &ctl->empty[stage]);
+          } else {
+            // Last, partial stage: only the K slices that hold features.
+            for (int kk = 0; kk < BK / 16 && kb * BK + kk * 16 < dim; ++kk) {
+              // K = 16 slice kk: swizzle atom kk / 4, 32 bytes per slice within it.
+              const uint64_t off = static_cast<uint64_t>((kk / 4) * (ATOM_BYTES >> 4) + (kk % 4) * 2);
+              mma_pair(d_tmem, a_desc + off, a_desc + (SLICE_BYTES >> 4) + off, IDESC, (kb | kk) != 0 ? 1u : 0u);
+            }
+            commit_both(&ctl->empty[stage]);
+          }
           if (++stage == STAGES) {
             stage = 0;
             phase ^= 1u;
@@ -434,7 +489,7 @@ cudaError_t launch_affinity_pair(const void* tokens, int batch, int64_t rows, in
   CUtensorMap map;
   const cuuint64_t gdim[2] = {static_cast<cuuint64_t>(dim), static_cast<cuuint64_t>(rows)};
   const cuuint64_t gstride[1] = {static_cast<cuuint64_t>(dim) * 2};
-  const cuuint32_t box[2] = {BK, HALF};
+  const cuuint32_t box[2] = {BOX_K, HALF};
   const cuuint32_t estride[2] = {1, 1};
   if (encode(&map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(tokens), gdim, gstride, box, estride,
              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -451,7 +506,6 @@ cudaError_t launch_affinity_pair(const void* tokens, int batch, int64_t rows, in
     if (e != cudaSuccess) return e;
     attr_done.fetch_or(bit);
   }
-  const int ksteps = (dim + BK - 1) / BK;
   const int grid = (num_sms > 1 ? num_sms : 2) & ~1;  // whole SM pairs
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
@@ -467,7 +521,7 @@ cudaError_t launch_affinity_pair(const void* tokens, int batch, int64_t rows, in
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, affinity_pair_kernel, map, batch, ksteps, ws);
+  return cudaLaunchKernelEx(&cfg, affinity_pair_kernel, map, batch, dim, ws);
 }
 
 }  // namespace mpm
