@@ -123,10 +123,7 @@ __device__ __forceinline__ unsigned long long column_candidate(const uint2* scra
 // A warp's whole COLS-column slice of one accumulator (TMEM columns
 // taddr .. taddr + COLS - 1, tile columns c0 ..), read in 16-column pieces
 // with the next piece's load in flight while the current one is processed.
-// The loop body covers two pieces (32 columns) and is not unrolled further,
-// which keeps the epilogue's code small: the MMA-issuing warp shares its
-// sub-partition's instruction cache with four epilogue warps.  Row
-// candidates use two independent running maxima (even and odd columns),
+// The loop body covers two pieces (32 columns).  Row candidates use two independent running maxima (even and odd columns),
 // merged at the end with the lowest-index rule, to halve the dependent
 // chain.  colcand[h] receives the column candidate of tile column
 // c0 + 32 h + lane (0 when none).
@@ -140,7 +137,7 @@ __device__ __forceinline__ void epilogue_slice(uint32_t taddr, const float* sc, 
   uint32_t va[16], vb[16];
   ptx::tmem_ld_32x32b_x16(taddr, va);
   ptx::tmem_wait_ld(va);
-#pragma unroll 1
+#pragma unroll
   for (int h = 0; h < COLS / 32; ++h) {
     const int c = c0 + 32 * h;
     ptx::tmem_ld_32x32b_x16(taddr + 32 * h + 16, vb);

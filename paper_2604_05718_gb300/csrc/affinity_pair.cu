@@ -24,11 +24,11 @@
 //    symmetric mode; the block below the diagonal of a diagonal tile is
 //    skipped.
 //
-// Roles per CTA (18 warps): warp 0 loads its CTA's A and B slices with TMA
+// Roles per CTA (10 warps): warp 0 loads its CTA's A and B slices with TMA
 // and reports the bytes to the leader CTA's barrier; in the leader, warp 1
 // allocates tensor memory (jointly with the peer) and issues the MMAs, whose
-// completion is multicast to both CTAs; warps 2-17 of each CTA read their own
-// tensor memory in 32 x 64 slices.  Every wait is bounded; on expiry the
+// completion is multicast to both CTAs; warps 2-9 of each CTA read their own
+// tensor memory in 32 x 128 slices.  Every wait is bounded; on expiry the
 // kernel records MPM_ERR_DEVICE_TIMEOUT and unwinds.
 #include <cuda.h>
 #include <cudaTypedefs.h>
@@ -53,8 +53,12 @@ constexpr int ATOM_BYTES = HALF * BOX_K * 2;   // 16 KiB
 constexpr int STAGES = 3;
 constexpr int SLICE_BYTES = ATOMS * ATOM_BYTES;  // 32 KiB: 128 rows x BK features
 constexpr int STAGE_BYTES = 2 * SLICE_BYTES;     // A slice + B slice of this CTA
-constexpr int EPI_WARPS = 16;
+// Epilogue warps: two per SM sub-partition, each reading 32 TMEM lanes x 128
+// columns.  Fewer, longer epilogue warps leave the MMA-issuing warp more of
+// its sub-partition's issue slots (measured: 8 warps beat 16 and 4).
+constexpr int EPI_WARPS = 8;
 constexpr int EPI_COLS = TILE / (EPI_WARPS / 4);
+static_assert(EPI_COLS <= HALF && HALF % EPI_COLS == 0, "a warp's columns lie in one 128-column block");
 constexpr int THREADS = (2 + EPI_WARPS) * 32;
 constexpr uint32_t TMEM_COLS = 2 * TILE;
 constexpr uint32_t IDESC = ptx::idesc_bf16_f32(2 * HALF, TILE);
@@ -380,8 +384,8 @@ __global__ void __launch_bounds__(THREADS, 1)
   } else {
     // ---------------- epilogue (both CTAs) ----------------
     // Warp (q, quarter) reads tile rows 32q..32q+31 of this CTA and tile
-    // columns c0..c0+63.  It keeps its own copy of those 64 column scales, so
-    // no epilogue warp ever waits for another one.
+    // columns c0..c0+EPI_COLS-1.  It keeps its own copy of those column
+    // scales, so no epilogue warp ever waits for another one.
     const int ew = warp - 2;
     const int q = warp & 3;
     const int quarter = ew >> 2;
@@ -392,12 +396,14 @@ __global__ void __launch_bounds__(THREADS, 1)
     uint2* scr = scratch_all + ew * 32;
     int acc = 0;
     uint32_t acc_phase = 0;
-    float pf_scale0 = 0.f, pf_scale1 = 0.f, pf_inv = 0.f;
+    float pf_scale[EPI_COLS / 32], pf_inv = 0.f;
     auto prefetch = [&](const Item& nx) {
       const float nan = __int_as_float(0x7fc00000);  // columns outside the image never win
-      const int j0 = nx.col0 + c0 + lane, j1 = j0 + 32;
-      pf_scale0 = j0 < nx.n ? __ldg(ws.inv_norm + nx.base + j0) : nan;
-      pf_scale1 = j1 < nx.n ? __ldg(ws.inv_norm + nx.base + j1) : nan;
+#pragma unroll
+      for (int h = 0; h < EPI_COLS / 32; ++h) {
+        const int j = nx.col0 + c0 + 32 * h + lane;
+        pf_scale[h] = j < nx.n ? __ldg(ws.inv_norm + nx.base + j) : nan;
+      }
       const int r = nx.row0 + HALF * static_cast<int>(rank) + q * 32 + lane;
       const bool col = (nx.col0 + c0) / HALF > (nx.row0 + HALF * static_cast<int>(rank)) / HALF;
       pf_inv = (col && r < nx.n) ? __ldg(ws.inv_norm + nx.base + r) : 0.f;
@@ -407,8 +413,8 @@ __global__ void __launch_bounds__(THREADS, 1)
     if (count > 0) prefetch(item(0));
     for (int64_t k = 0; k < count; ++k) {
       const Item it = item(k);
-      my_scale[lane] = pf_scale0;
-      my_scale[lane + 32] = pf_scale1;
+#pragma unroll
+      for (int h = 0; h < EPI_COLS / 32; ++h) my_scale[32 * h + lane] = pf_scale[h];
       const float inv_i = pf_inv;
       __syncwarp();
       if (!ptx::mbar_wait(&ctl->acc_full[acc], acc_phase, abort_flag, WAIT_LIMIT_NS)) {
