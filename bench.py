@@ -45,7 +45,10 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 L2_FLUSH_BYTES = 256 << 20
 KERNELS_PER_MERGE = 4
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "affinity_pair_traffic.txt")
-AFFINITY_SOURCE = os.path.join(ROOT, "paper_2604_05718_gb300", "csrc", "affinity_pair.cu")
+# The sources the affinity kernel is compiled from; the traffic record holds
+# a hash of their concatenation.
+AFFINITY_SOURCES = [os.path.join(ROOT, "paper_2604_05718_gb300", "csrc", f)
+                    for f in ("affinity_pair.cu", "affinity_epilogue.cuh", "ptx.cuh", "common.cuh")]
 
 
 def parse_args():
@@ -274,7 +277,16 @@ class ClockSampler:
                 "samples": len(sm), "source": "NVML, 1 ms period, during the timed steps"}
 
 
-def traffic_for(kernel_file: str, rows_per_launch: float):
+def kernel_sources_sha(files) -> str:
+    """First 16 hex digits of the SHA-256 of the files' concatenated bytes."""
+    h = hashlib.sha256()
+    for name in files:
+        with open(name, "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def traffic_for(kernel_files, rows_per_launch: float):
     """DRAM bytes per launch from the committed ncu record, if the kernel is unchanged.
 
     The record holds one captured launch's dram read + write bytes and its
@@ -283,9 +295,7 @@ def traffic_for(kernel_file: str, rows_per_launch: float):
     try:
         with open(TRAFFIC_FILE) as f:
             fields = dict(line.strip().split("=", 1) for line in f if "=" in line and not line.startswith("#"))
-        with open(kernel_file, "rb") as f:
-            sha = hashlib.sha256(f.read()).hexdigest()[:16]
-        if fields.get("source_sha256_16") == sha:
+        if fields.get("source_sha256_16") == kernel_sources_sha(kernel_files):
             per_row = (float(fields["dram_read_bytes"]) + float(fields["dram_write_bytes"])) / \
                 float(fields["rows_captured"])
             return per_row * rows_per_launch
@@ -480,7 +490,7 @@ def run_mpm(args):
     exe = [exec_flops(n0)] * args.steps + ([exec_flops(n1)] * args.steps if two else [])
     executed_tflops = sum(exe) / (sum(aff_ms) * 1e-3) / 1e12
     rows_per_launch = (n0.sum() + (n1.sum() if two else 0.0)) / (2.0 if two else 1.0)
-    traffic = traffic_for(AFFINITY_SOURCE, rows_per_launch)
+    traffic = traffic_for(AFFINITY_SOURCES, rows_per_launch)
     roofline = {
         "kernel": "affinity_pair_kernel (fused cosine affinity + arg max, TMA + tcgen05.mma.cta_group::2)",
         "bound": "tensor", "achieved": achieved_tflops, "peak": tensor_peak, "unit": "TFLOP/s",
