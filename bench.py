@@ -372,7 +372,7 @@ def run_mpm(args):
             self.seg = new_events(4)       # [merge1 start, merge1 end, rest start, rest end]
             self.k1 = new_events(8)        # merge 1 kernels
             self.k2 = new_events(8)        # merge 2 kernels
-            self.cg = new_events(2)        # between compose and gather
+            self.cg = new_events(2)        # around the (composed) gather
 
     def step(ev: StepEvents, host_in=None, host_out=None, per_kernel=False):
         """One step; per_kernel adds CUDA events between the kernels (which
@@ -394,10 +394,10 @@ def run_mpm(args):
         if two:
             mpm.merge(x1n, off1, workspace=ws, out_tokens=x2, out_offsets=off2, out_map=m2,
                       stage_events=ev.k2 if per_kernel else None)
-            mpm.compose_maps(m1, off0, m2, off1, out=rstar)
             if per_kernel:
                 ev.cg[0].record(stream)
-            mpm.unmerge_gather(x2, off2, rstar, off0, out=up)
+            # Eq. 3 and Eq. 4 in one pass; rstar receives the composed map.
+            mpm.compose_gather(x2, off2, m1, off0, m2, off1, out=up, out_map=rstar)
         else:
             if per_kernel:
                 ev.cg[0].record(stream)
@@ -462,7 +462,7 @@ def run_mpm(args):
         if two:
             kern[f"{nm}_2_us"] = 1e3 * statistics.mean(kernel_ms("k2", k))
     cg = [ev.cg[0].elapsed_time(ev.cg[1]) for ev in kevents]
-    kern["gather_us"] = 1e3 * statistics.mean(cg)
+    kern["gather_us" if not two else "compose_gather_us"] = 1e3 * statistics.mean(cg)
 
     peaks, peak_kind = load_peaks()
     n0 = np.diff(batch.offsets).astype(np.float64)
@@ -507,11 +507,13 @@ def run_mpm(args):
     # HBM fractions of the bandwidth kernels (algorithmic bytes / event time).
     hbm = peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
     avg1 = float((n0.sum() + n1.sum()) * dim * esize + 12 * n0.sum())
-    gat = float((n2.sum() + n0.sum()) * dim * esize + 4 * n0.sum())
+    # Gather reads each merged row it needs and writes the grid; with two
+    # insertions it also reads both maps and writes the composed one.
+    gat = float((n2.sum() + n0.sum()) * dim * esize + (12 if two else 4) * n0.sum())
     norm1 = float(n0.sum() * dim * esize + 12 * n0.sum())
     hbm_kernels = {
         "pair_average_1_gbs": avg1 / (kern["pair_average_1_us"] * 1e-6) / 1e9,
-        "gather_gbs": gat / (kern["gather_us"] * 1e-6) / 1e9,
+        "gather_gbs": gat / (kern["gather_us" if not two else "compose_gather_us"] * 1e-6) / 1e9,
         "prep_1_gbs": norm1 / (kern["prep_1_us"] * 1e-6) / 1e9,
         "peak_gbs": hbm, "peak_kind": f"{peak_kind} copy bandwidth",
     }
@@ -558,8 +560,7 @@ def run_mpm(args):
                 if two:
                     x1n[:t1] = apply_noise(x1[:t1], noise)
                     mpm.merge(x1n, off1, workspace=ws, out_tokens=x2, out_offsets=off2, out_map=m2)
-                    mpm.compose_maps(m1, dev_off[sl], m2, off1, out=rstar)
-                    mpm.unmerge_gather(x2, off2, rstar, dev_off[sl], out=dev_up[sl])
+                    mpm.compose_gather(x2, off2, m1, dev_off[sl], m2, off1, out=dev_up[sl], out_map=rstar)
                 else:
                     mpm.unmerge_gather(x1, off1, m1, dev_off[sl], out=dev_up[sl])
                 inputs_free[sl].record(stream)
@@ -607,7 +608,7 @@ def run_mpm(args):
             "cpu_baseline": cpu_base,
             "e2e": e2e,
             "clocks": clk,
-            "gpu_launches": (2 * KERNELS_PER_MERGE + 2 if two else KERNELS_PER_MERGE + 1) * args.steps,
+            "gpu_launches": (2 * KERNELS_PER_MERGE + 1 if two else KERNELS_PER_MERGE + 1) * args.steps,
             "wall_s_timed_loop": wall,
         }
         print(json.dumps(line), flush=True)

@@ -204,6 +204,31 @@ MPM_API mpm_status mpm_unmerge_gather(const void* merged, const int64_t* merged_
                               int32_t* device_status, void* stream);
 
 /*
+ * Composition and gather in one pass (Eq. 3 then Eq. 4), for two
+ * insertions: for every grid row p of image b,
+ *   r*(p) = map2[offsets1_b + map1[p]]   and   out[p] = merged[m_b + r*(p)].
+ * The result equals mpm_compose_maps followed by mpm_unmerge_gather, without
+ * the separate pass over the composed map.
+ *
+ *   merged          [merged_rows, dim] stage-2 tokens (dtype); merged_offsets
+ *                   int64 [batch + 1] their images
+ *   map1, offsets0  int32 [rows0] stage-1 map and int64 [batch + 1] grid images
+ *   map2, offsets1  int32 [rows1] stage-2 map and int64 [batch + 1] stage-1 images
+ *   out             [rows0, dim] (dtype), written for rows < offsets0[batch]
+ *   out_map         optional int32 [rows0]: receives r* (may alias map1, not
+ *                   map2); NULL when the composed map is not wanted
+ *   device_status   optional int32 device word; an out-of-range entry of either
+ *                   map zeroes that output row, writes -1 to out_map there and
+ *                   records MPM_ERR_DEVICE_CHECK.
+ * out must not overlap merged (MPM_ERR_ALIASING).
+ */
+MPM_API mpm_status mpm_compose_gather(const void* merged, const int64_t* merged_offsets,
+                              int64_t merged_rows, const int32_t* map1, const int64_t* offsets0,
+                              int64_t rows0, const int32_t* map2, const int64_t* offsets1,
+                              int64_t rows1, int32_t batch, int32_t dim, mpm_dtype dtype,
+                              void* out, int32_t* out_map, int32_t* device_status, void* stream);
+
+/*
  * Nearest neighbours only (Eq. 1 and Algorithm 1 step 3), for testing and
  * diagnostics.  out_nn int32 [rows]: local index b(i) (-1 for a token alone
  * in its image); out_score float [rows] (may be NULL): the cosine S_{i,b(i)}

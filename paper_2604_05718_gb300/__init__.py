@@ -7,6 +7,7 @@ marshals torch tensors into its C entry points.
 
 from .mpm import (  # noqa: F401
     MPMError,
+    compose_gather,
     compose_maps,
     device_status,
     library,

@@ -303,15 +303,23 @@ __global__ void compose_kernel(const int32_t* map1, const int64_t* __restrict__ 
 }
 
 // ---------------------------------------------------------------------------
-// Gather reconstruction (Eq. 4): one warp per grid row, pure copy.
+// Gather reconstruction (Eq. 4), a pure copy.  A warp takes 32 consecutive
+// grid rows: lane l resolves row p0 + l (its image, its map entry and the
+// source row, all independent loads across the lanes), then the warp copies
+// the rows RG at a time with every lane moving 16-byte vectors.  With
+// COMPOSE the source is composed on the way (Eq. 3):
+// r*(p) = map2[off1_b + map1[p]], and r* is written to out_map if given.
 // ---------------------------------------------------------------------------
-template <int U>
+template <int U, int RG, bool COMPOSE>
 __global__ void __launch_bounds__(kThreads) gather_kernel(const uint8_t* __restrict__ merged,
                                                           const int64_t* __restrict__ moff,
                                                           int64_t merged_rows,
-                                                          const int32_t* __restrict__ map,
+                                                          const int32_t* map,
                                                           const int64_t* __restrict__ goff,
-                                                          int64_t grid_rows, int batch, int row_bytes,
+                                                          int64_t grid_rows,
+                                                          const int32_t* __restrict__ map2,
+                                                          const int64_t* __restrict__ off1, int64_t rows1,
+                                                          int32_t* out_map, int batch, int row_bytes,
                                                           uint8_t* __restrict__ out, int32_t* status) {
   wait_for_previous_grid();
   const int lane = threadIdx.x & 31;
@@ -320,26 +328,51 @@ __global__ void __launch_bounds__(kThreads) gather_kernel(const uint8_t* __restr
   const int64_t used = clamp64(goff[batch], 0, grid_rows);
   const int nvec = row_bytes >> 4;
   ImageCursor cur;
-  for (int64_t p = warp; p < used; p += nwarps) {
-    cur.locate(goff, batch, p);
-    const int64_t mlo = __ldg(moff + cur.b), mhi = __ldg(moff + cur.b + 1);
-    const int32_t m = __ldg(map + p);
-    const bool ok = p >= cur.lo && p < cur.hi && m >= 0 && m < mhi - mlo && mlo >= 0 &&
-                    mlo + m < merged_rows;
-    if (!ok && lane == 0) report(status, MPM_ERR_DEVICE_CHECK, static_cast<int32_t>(p));
-    const uint4* src = reinterpret_cast<const uint4*>(merged + (ok ? (mlo + m) : 0) * row_bytes);
-    uint4* dst = reinterpret_cast<uint4*>(out + p * row_bytes);
-    for (int v0 = lane; v0 < nvec; v0 += 32 * U) {
-      uint4 val[U];
-#pragma unroll
-      for (int u = 0; u < U; ++u) {
-        const int v = v0 + 32 * u;
-        if (v < nvec) val[u] = ok ? __ldg(src + v) : make_uint4(0, 0, 0, 0);
+  for (int64_t p0 = warp * 32; p0 < used; p0 += nwarps * 32) {
+    // Lane l resolves grid row p0 + l.
+    const int64_t p = p0 + lane;
+    int64_t src = -1;  // merged row to copy, -1 = none (zero row)
+    if (p < used) {
+      cur.locate(goff, batch, p);
+      const int64_t mlo = __ldg(moff + cur.b), mhi = __ldg(moff + cur.b + 1);
+      int32_t m = map[p];
+      bool ok = p >= cur.lo && p < cur.hi;
+      if (COMPOSE) {
+        // Stage-1 index of this grid row, then its stage-2 (merged) index.
+        const int64_t lo1 = __ldg(off1 + cur.b), hi1 = __ldg(off1 + cur.b + 1);
+        ok = ok && m >= 0 && m < hi1 - lo1 && lo1 >= 0 && lo1 + m < rows1;
+        m = ok ? __ldg(map2 + lo1 + m) : -1;
       }
+      ok = ok && m >= 0 && m < mhi - mlo && mlo >= 0 && mlo + m < merged_rows;
+      if (!ok) report(status, MPM_ERR_DEVICE_CHECK, static_cast<int32_t>(p));
+      // This lane alone reads and writes entry p, so out_map may alias map.
+      if (COMPOSE && out_map != nullptr) out_map[p] = ok ? m : -1;
+      src = ok ? mlo + m : -1;
+    }
+    const int nrows = static_cast<int>(used - p0 < 32 ? used - p0 : 32);
+    for (int r0 = 0; r0 < nrows; r0 += RG) {
+      int64_t s[RG];
 #pragma unroll
-      for (int u = 0; u < U; ++u) {
-        const int v = v0 + 32 * u;
-        if (v < nvec) __stcs(dst + v, val[u]);
+      for (int g = 0; g < RG; ++g) s[g] = __shfl_sync(0xFFFFFFFFu, src, (r0 + g) & 31);
+      for (int v0 = lane; v0 < nvec; v0 += 32 * U) {
+        uint4 val[RG][U];
+#pragma unroll
+        for (int g = 0; g < RG; ++g)
+#pragma unroll
+          for (int u = 0; u < U; ++u) {
+            const int v = v0 + 32 * u;
+            if (r0 + g < nrows && v < nvec)
+              val[g][u] = s[g] >= 0 ? __ldg(reinterpret_cast<const uint4*>(merged + s[g] * row_bytes) + v)
+                                    : make_uint4(0, 0, 0, 0);
+          }
+#pragma unroll
+        for (int g = 0; g < RG; ++g)
+#pragma unroll
+          for (int u = 0; u < U; ++u) {
+            const int v = v0 + 32 * u;
+            if (r0 + g < nrows && v < nvec)
+              __stcs(reinterpret_cast<uint4*>(out + (p0 + r0 + g) * row_bytes) + v, val[g][u]);
+          }
       }
     }
   }
@@ -391,9 +424,22 @@ cudaError_t launch_gather(const void* merged, const int64_t* moff, int64_t merge
                           int dim, bool bf16, void* out, int32_t* status, int num_sms,
                           cudaStream_t stream) {
   const int row_bytes = dim * (bf16 ? 2 : 4);
-  return launch_dependent(gather_kernel<4>, dim3(grid_for(num_sms, 8)), dim3(kThreads), 0, stream,
-                          static_cast<const uint8_t*>(merged), moff, merged_rows, map, goff, grid_rows, batch,
-                          row_bytes, static_cast<uint8_t*>(out), status);
+  return launch_dependent(gather_kernel<3, 4, false>, dim3(grid_for(num_sms, 8)), dim3(kThreads), 0, stream,
+                          static_cast<const uint8_t*>(merged), moff, merged_rows, map, goff, grid_rows,
+                          static_cast<const int32_t*>(nullptr), static_cast<const int64_t*>(nullptr),
+                          static_cast<int64_t>(0), static_cast<int32_t*>(nullptr), batch, row_bytes,
+                          static_cast<uint8_t*>(out), status);
+}
+
+cudaError_t launch_compose_gather(const void* merged, const int64_t* moff, int64_t merged_rows,
+                                  const int32_t* map1, const int64_t* off0, int64_t rows0,
+                                  const int32_t* map2, const int64_t* off1, int64_t rows1, int batch, int dim,
+                                  bool bf16, void* out, int32_t* out_map, int32_t* status, int num_sms,
+                                  cudaStream_t stream) {
+  const int row_bytes = dim * (bf16 ? 2 : 4);
+  return launch_dependent(gather_kernel<3, 4, true>, dim3(grid_for(num_sms, 8)), dim3(kThreads), 0, stream,
+                          static_cast<const uint8_t*>(merged), moff, merged_rows, map1, off0, rows0, map2, off1,
+                          rows1, out_map, batch, row_bytes, static_cast<uint8_t*>(out), status);
 }
 
 }  // namespace mpm

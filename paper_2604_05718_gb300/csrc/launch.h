@@ -78,4 +78,11 @@ cudaError_t launch_gather(const void* merged, const int64_t* moff, int64_t merge
                           int dim, bool bf16, void* out, int32_t* status, int num_sms,
                           cudaStream_t stream);
 
+// Composition (Eq. 3) and gather (Eq. 4) in one pass over the grid rows.
+cudaError_t launch_compose_gather(const void* merged, const int64_t* moff, int64_t merged_rows,
+                                  const int32_t* map1, const int64_t* off0, int64_t rows0,
+                                  const int32_t* map2, const int64_t* off1, int64_t rows1, int batch, int dim,
+                                  bool bf16, void* out, int32_t* out_map, int32_t* status, int num_sms,
+                                  cudaStream_t stream);
+
 }  // namespace mpm

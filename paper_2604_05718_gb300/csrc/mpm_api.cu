@@ -262,6 +262,29 @@ mpm_status mpm_unmerge_gather(const void* merged, const int64_t* merged_offsets,
                                         static_cast<cudaStream_t>(stream)));
 }
 
+mpm_status mpm_compose_gather(const void* merged, const int64_t* merged_offsets, int64_t merged_rows,
+                              const int32_t* map1, const int64_t* offsets0, int64_t rows0, const int32_t* map2,
+                              const int64_t* offsets1, int64_t rows1, int32_t batch, int32_t dim, mpm_dtype dtype,
+                              void* out, int32_t* out_map, int32_t* device_status, void* stream) {
+  if (!sizes_ok(merged_rows, batch) || !sizes_ok(rows0, batch) || !sizes_ok(rows1, batch) ||
+      merged_offsets == nullptr || offsets0 == nullptr || offsets1 == nullptr)
+    return MPM_ERR_INVALID_ARG;
+  mpm_status st = check_tokens(merged, merged_rows, dim, dtype);
+  if (st != MPM_OK) return st;
+  if (rows0 == 0) return MPM_OK;
+  if (map1 == nullptr || out == nullptr || (map2 == nullptr && rows1 > 0)) return MPM_ERR_INVALID_ARG;
+  if (!aligned16(out)) return MPM_ERR_ALIGNMENT;
+  const size_t row_bytes = static_cast<size_t>(dim) * elem_size(dtype);
+  if (overlap(merged, row_bytes * merged_rows, out, row_bytes * rows0)) return MPM_ERR_ALIASING;
+  if (out_map != nullptr && overlap(out_map, sizeof(int32_t) * rows0, map2, sizeof(int32_t) * rows1))
+    return MPM_ERR_ALIASING;
+  const int sms = num_sms();
+  if (sms <= 0) return MPM_ERR_CUDA;
+  return cuda_status(mpm::launch_compose_gather(merged, merged_offsets, merged_rows, map1, offsets0, rows0, map2,
+                                                offsets1, rows1, batch, dim, dtype == MPM_BF16, out, out_map,
+                                                device_status, sms, static_cast<cudaStream_t>(stream)));
+}
+
 mpm_status mpm_get_device_status(void* workspace, int32_t* host_code, void* stream) {
   if (workspace == nullptr || host_code == nullptr) return MPM_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);

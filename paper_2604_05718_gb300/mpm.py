@@ -28,7 +28,7 @@ STATUS_NAMES = {
 }
 EXPORTS = ("mpm_abi_version", "mpm_status_string", "mpm_merge_workspace_size", "mpm_merge", "mpm_merge_timed",
            "mpm_compose_maps", "mpm_unmerge_gather", "mpm_nearest_neighbors", "mpm_get_device_status",
-           "mpm_merge_no_alloc")
+           "mpm_merge_no_alloc", "mpm_compose_gather")
 
 _lib = None
 
@@ -55,6 +55,8 @@ def _declare(lib: ctypes.CDLL) -> None:
                                                  SZ, P]),
         "mpm_get_device_status": (ctypes.c_int, [P, P, P]),
         "mpm_merge_no_alloc": (ctypes.c_int, [P, P, I32, I64, I32, ctypes.c_int, P, P, P, P]),
+        "mpm_compose_gather": (ctypes.c_int, [P, P, I64, P, P, I64, P, P, I64, I32, I32, ctypes.c_int, P, P, P,
+                                              P]),
     }
     for name, (res, args) in sigs.items():
         fn = getattr(lib, name)
@@ -218,6 +220,37 @@ def unmerge_gather(merged: torch.Tensor, merged_offsets: torch.Tensor, rmap: tor
                                             merged.shape[1], _dtype_code(merged), _ptr(out),
                                             _ptr(device_status), _stream(dev))
     _check("mpm_unmerge_gather", code)
+    return out
+
+
+def compose_gather(merged: torch.Tensor, merged_offsets: torch.Tensor, map1: torch.Tensor,
+                   offsets0: torch.Tensor, map2: torch.Tensor, offsets1: torch.Tensor,
+                   out: torch.Tensor | None = None, out_map: torch.Tensor | None = None,
+                   device_status: torch.Tensor | None = None) -> torch.Tensor:
+    """Eq. 3 and Eq. 4 in one pass: out[p] = merged[r2(r1(p))] per image.
+
+    out has map1.numel() rows; out_map, if given, receives the composed map.
+    """
+    _cuda(merged, "merged", ndim=2)
+    _cuda(merged_offsets, "merged_offsets", torch.int64, 1)
+    _cuda(map1, "map1", torch.int32, 1)
+    _cuda(offsets0, "offsets0", torch.int64, 1)
+    _cuda(map2, "map2", torch.int32, 1)
+    _cuda(offsets1, "offsets1", torch.int64, 1)
+    if out_map is not None:
+        _cuda(out_map, "out_map", torch.int32, 1)
+        if out_map.numel() < map1.numel():
+            raise ValueError("out_map needs map1.numel() entries")
+    dev = merged.device
+    if out is None:
+        out = torch.empty(map1.numel(), merged.shape[1], dtype=merged.dtype, device=dev)
+    with torch.cuda.device(dev):
+        code = library().mpm_compose_gather(_ptr(merged), _ptr(merged_offsets), merged.shape[0], _ptr(map1),
+                                            _ptr(offsets0), out.shape[0], _ptr(map2), _ptr(offsets1),
+                                            map2.numel(), offsets0.numel() - 1, merged.shape[1],
+                                            _dtype_code(merged), _ptr(out), _ptr(out_map),
+                                            _ptr(device_status), _stream(dev))
+    _check("mpm_compose_gather", code)
     return out
 
 

@@ -111,4 +111,17 @@ def test_nn_compose_gather_validation(lib):
     assert gat(P(FAKE), P(FAKE), 10, P(FAKE), P(FAKE), 10, 1, 64, 1, None, None, None) == 1
     assert gat(P(FAKE), P(FAKE), 10, P(FAKE), P(FAKE), 10, 1, 64, 1, P(FAKE + 128), None, None) == 8
     assert gat(P(FAKE), P(FAKE), 10, P(FAKE), P(FAKE), 10, 1, 60, 1, P(FAKE * 8), None, None) == 3
+    cg = lib.mpm_compose_gather
+    # (merged, merged_offsets, merged_rows, map1, offsets0, rows0, map2, offsets1, rows1, batch, dim, dtype,
+    #  out, out_map, device_status, stream)
+    assert cg(P(FAKE), None, 10, P(FAKE), P(FAKE), 10, P(FAKE), P(FAKE), 10, 1, 64, 1, P(FAKE * 8), None, None,
+              None) == 1                                                                   # no merged offsets
+    assert cg(P(FAKE), P(FAKE), 10, P(FAKE), P(FAKE), 10, P(FAKE), P(FAKE), 10, 1, 64, 1, None, None, None,
+              None) == 1                                                                   # no output
+    assert cg(P(FAKE), P(FAKE), 10, P(FAKE), P(FAKE), 10, P(FAKE), P(FAKE), 10, 1, 64, 1, P(FAKE + 128), None,
+              None, None) == 8                                                             # out overlaps merged
+    assert cg(P(FAKE), P(FAKE), 10, P(FAKE), P(FAKE), 10, P(FAKE * 4), P(FAKE), 10, 1, 64, 1, P(FAKE * 8),
+              P(FAKE * 4 + 8), None, None) == 8                                            # out_map overlaps map2
+    assert cg(P(FAKE), P(FAKE), 10, P(FAKE), P(FAKE), 10, P(FAKE), P(FAKE), 10, 1, 60, 1, P(FAKE * 8), None,
+              None, None) == 3                                                             # rows not 16-byte multiples
     assert lib.mpm_get_device_status(None, None, None) == 1

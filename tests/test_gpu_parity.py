@@ -208,6 +208,17 @@ def test_compose_and_gather_kernels_on_oracle_maps(mpm, dtype):
     up = mpm.unmerge_gather(z, i64(o2.out_offsets), i32(r_star), i64(batch.offsets), device_status=status)
     want = oracle.gather_batch(z.double().cpu().numpy(), o2.out_offsets, r_star, batch.offsets)
     assert np.array_equal(to_f64(up), want)
+    # Eq. 3 and Eq. 4 fused: the same grid and the same composed map, also in place over map1.
+    rmap = torch.full((batch.rows,), -7, dtype=torch.int32, device=DEV)
+    fused = mpm.compose_gather(z, i64(o2.out_offsets), i32(o1.r), i64(batch.offsets), i32(o2.r),
+                               i64(o1.out_offsets), out_map=rmap, device_status=status)
+    assert np.array_equal(to_f64(fused), want)
+    assert np.array_equal(rmap.cpu().numpy(), r_star)
+    inplace = i32(o1.r)
+    fused2 = mpm.compose_gather(z, i64(o2.out_offsets), inplace, i64(batch.offsets), i32(o2.r),
+                                i64(o1.out_offsets), out_map=inplace, device_status=status)
+    assert np.array_equal(inplace.cpu().numpy(), r_star)
+    assert torch.equal(fused2, fused)
     assert int(status[0]) == 0
 
 
