@@ -520,6 +520,41 @@ def run_mpm(args):
     for k in ("pair_average_1", "gather", "prep_1"):
         hbm_kernels[k + "_frac"] = hbm_kernels[k + "_gbs"] / hbm
 
+    # ---------------- padded batch of the stage-1 output (next-step consumer layout) ----------------
+    # The merged sequences padded to the longest one, with a key mask, as the
+    # paper batches them for dense attention; and back to the packed layout.
+    n1_max = int(n1.max())
+    pad_out = torch.empty(nimg, n1_max, dim, dtype=x1.dtype, device=dev)
+    pad_mask = torch.empty(nimg, n1_max, dtype=torch.uint8, device=dev)
+    pad_stats = torch.empty(3, dtype=torch.int64, device=dev)
+    unpadded = torch.empty_like(x1)
+    pad_us, unpad_us = [], []
+    for it in range(max(3, args.warmup) + 20):
+        flush.fill_(1)
+        flush_sum.copy_(flush.view(torch.int64).sum())
+        e = new_events(3)
+        e[0].record(stream)
+        mpm.pad_batch(x1, off1, n1_max, out=pad_out, mask=pad_mask, stats=pad_stats)
+        e[1].record(stream)
+        mpm.unpad_batch(pad_out, off1, out=unpadded)
+        e[2].record(stream)
+        if it >= max(3, args.warmup):
+            torch.cuda.synchronize(dev)
+            pad_us.append(1e3 * e[0].elapsed_time(e[1]))
+            unpad_us.append(1e3 * e[1].elapsed_time(e[2]))
+    assert torch.equal(unpadded[:t1], x1[:t1]), "unpad(pad(x)) differs from x"
+    hbm_bw = peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
+    pad_bytes = float(n1.sum() * dim * esize + nimg * n1_max * (dim * esize + 1))
+    unpad_bytes = float(2 * n1.sum() * dim * esize)
+    padded = {
+        "L": n1_max, "rows": int(n1.sum()), "padding_frac": 1.0 - float(n1.sum()) / (nimg * n1_max),
+        "pad_us": statistics.median(pad_us), "unpad_us": statistics.median(unpad_us),
+        "pad_gbs": pad_bytes / (statistics.median(pad_us) * 1e-6) / 1e9,
+        "unpad_gbs": unpad_bytes / (statistics.median(unpad_us) * 1e-6) / 1e9,
+    }
+    padded["pad_frac"] = padded["pad_gbs"] / hbm_bw
+    padded["unpad_frac"] = padded["unpad_gbs"] / hbm_bw
+
     # ---------------- end to end: host buffers, copies inside the timed region ----------------
     # A serving loop: every step copies its tokens and offsets in from pinned
     # host memory, runs the whole step (L2 flush, merge, stand-in noise,
@@ -603,6 +638,7 @@ def run_mpm(args):
             "merged_tokens": {"stage0": int(n0.sum()), "stage1": int(n1.sum()), "stage2": int(n2.sum())},
             "roofline": roofline,
             "hbm_kernels": hbm_kernels,
+            "padded_batch": padded,
             "kernels_us": kern,
             "ms_per_step_with_kernel_events": ms_with_kernel_events,
             "cpu_baseline": cpu_base,

@@ -229,6 +229,47 @@ MPM_API mpm_status mpm_compose_gather(const void* merged, const int64_t* merged_
                               void* out, int32_t* out_map, int32_t* device_status, void* stream);
 
 /*
+ * Padded batch for dense-attention consumers.  Section 4 (Analyses) batches
+ * images by padding each to the batch's longest merged sequence; a key mask
+ * keeps the padding out of attention.  The paper prints no routine for this
+ * step; the definition is:
+ *   out[b, t]     = tokens[offsets[b] + t]  for t < min(N_b, max_len), else a zero row
+ *   out_mask[b,t] = 1 for the copied rows, 0 for padding
+ * with N_b = offsets[b+1] - offsets[b].
+ *
+ *   tokens     [rows, dim] packed (dtype), offsets int64 [batch + 1] on the device
+ *   max_len    L >= 0, the padded length (e.g. the largest N_b, or the input
+ *              N as a bound the host knows without reading offsets)
+ *   out        [batch, L, dim] (dtype), 16-byte aligned, must not overlap tokens
+ *   out_mask   optional uint8 [batch, L]
+ *   out_stats  optional int64 [3]: min, max and total of N_b over the batch
+ *   device_status  optional int32 device word: an image longer than L is cut
+ *              to its first L rows and reported as MPM_ERR_DEVICE_CHECK
+ *              (detail = image index).
+ * All outputs are written on `stream`; nothing is read back to the host.
+ */
+MPM_API mpm_status mpm_pad_batch(const void* tokens, const int64_t* offsets, int32_t batch, int64_t rows,
+                                 int32_t dim, mpm_dtype dtype, int64_t max_len, void* out,
+                                 uint8_t* out_mask, int64_t* out_stats, int32_t* device_status,
+                                 void* stream);
+
+/*
+ * Inverse of mpm_pad_batch: out[offsets[b] + t] = padded[b, t] for
+ * t < N_b (N_b <= max_len), the packed layout the merge entry points take.
+ *
+ *   padded     [batch, max_len, dim] (dtype)
+ *   offsets    int64 [batch + 1]: the packed images; rows = capacity of out
+ *   out        [rows, dim] (dtype), written for rows < offsets[batch]; must
+ *              not overlap padded
+ *   device_status  optional: rows of an image longer than max_len are left
+ *              untouched and reported as MPM_ERR_DEVICE_CHECK (detail = image
+ *              index).
+ */
+MPM_API mpm_status mpm_unpad_batch(const void* padded, int32_t batch, int64_t max_len, int32_t dim,
+                                   mpm_dtype dtype, const int64_t* offsets, int64_t rows, void* out,
+                                   int32_t* device_status, void* stream);
+
+/*
  * Nearest neighbours only (Eq. 1 and Algorithm 1 step 3), for testing and
  * diagnostics.  out_nn int32 [rows]: local index b(i) (-1 for a token alone
  * in its image); out_score float [rows] (may be NULL): the cosine S_{i,b(i)}

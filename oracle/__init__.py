@@ -22,6 +22,8 @@ from .mpm_oracle import (  # noqa: F401
     mutual_partners,
     nearest_neighbours,
     normalise_rows,
+    pad_batch,
     round_bf16,
     round_f32,
+    unpad_batch,
 )

@@ -19,8 +19,10 @@ algorithm step (Section 3.2 "Mutual Pair Merging", Eq. 1-4, Algorithm 1):
   * ``merge_batch`` / ``compose_batch`` / ``gather_batch`` - the same steps
     applied image by image over a packed ragged batch ("batches are processed
     independently", Section 3.1).
+  * ``pad_batch`` / ``unpad_batch`` - the padded batch of Section 4
+    (Analyses): images padded to the longest merged sequence, with a key mask.
 
-Readings of points the paper leaves open (each also listed in the design doc):
+Readings of points the paper leaves open:
   * zero-norm rows are normalised by max(||x||, 1e-12) (Eq. 1 says only
     "L2-normalize");
   * ties in the arg max go to the lowest index j (the paper only says ties are
@@ -276,6 +278,42 @@ def gather_batch(z: np.ndarray, z_offsets: np.ndarray, r_star: np.ndarray,
         g0, g1 = grid_offsets[b], grid_offsets[b + 1]
         z0, z1 = z_offsets[b], z_offsets[b + 1]
         out[g0:g1] = gather(z[z0:z1], r_star[g0:g1])
+    return out
+
+
+# ---------------------------------------------------------------------------
+# Padded batches for dense-attention consumers (Section 4, Analyses: the
+# images of a batch are padded to the longest merged sequence, and the
+# padding is masked out of attention).
+# ---------------------------------------------------------------------------
+def pad_batch(x: np.ndarray, offsets: np.ndarray, max_len: int):
+    """Packed [T, d] tokens -> ([B, L, d] padded, [B, L] key mask, (min, max, total) of N_b).
+
+    Row t of image b is copied when t < min(N_b, L); every other row is zero and
+    masked out (mask 0).  An image longer than L is cut to its first L rows.
+    """
+    x = np.asarray(x)
+    offsets = np.asarray(offsets, dtype=np.int64)
+    batch = len(offsets) - 1
+    counts = offsets[1:] - offsets[:-1]
+    out = np.zeros((batch, max_len, x.shape[1]), dtype=x.dtype)
+    mask = np.zeros((batch, max_len), dtype=np.uint8)
+    for b in range(batch):
+        n = min(int(counts[b]), max_len)
+        out[b, :n] = x[offsets[b]:offsets[b] + n]
+        mask[b, :n] = 1
+    stats = (int(counts.min()) if batch else 0, int(counts.max()) if batch else 0, int(counts.sum()))
+    return out, mask, stats
+
+
+def unpad_batch(padded: np.ndarray, offsets: np.ndarray) -> np.ndarray:
+    """Inverse of pad_batch: packed row offsets[b] + t = padded[b, t] for t < N_b (N_b <= L)."""
+    padded = np.asarray(padded)
+    offsets = np.asarray(offsets, dtype=np.int64)
+    out = np.zeros((int(offsets[-1]), padded.shape[2]), dtype=padded.dtype)
+    for b in range(len(offsets) - 1):
+        n = int(offsets[b + 1] - offsets[b])
+        out[offsets[b]:offsets[b] + n] = padded[b, :n]
     return out
 
 

@@ -14,6 +14,8 @@ from .mpm import (  # noqa: F401
     merge,
     nearest_neighbors,
     new_workspace,
+    pad_batch,
     unmerge_gather,
+    unpad_batch,
     workspace_size,
 )

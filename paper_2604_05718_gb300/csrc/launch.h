@@ -85,4 +85,12 @@ cudaError_t launch_compose_gather(const void* merged, const int64_t* moff, int64
                                   bool bf16, void* out, int32_t* out_map, int32_t* status, int num_sms,
                                   cudaStream_t stream);
 
+// Padded batch [batch, max_len, dim] + key mask + N_b statistics, and its
+// inverse (kernels_pad.cu).
+cudaError_t launch_pad(const void* tokens, const int64_t* offsets, int batch, int64_t rows, int64_t max_len,
+                       int dim, bool bf16, void* out, uint8_t* mask, int64_t* stats, int32_t* status, int num_sms,
+                       cudaStream_t stream);
+cudaError_t launch_unpad(const void* padded, int batch, int64_t max_len, const int64_t* offsets, int64_t rows,
+                         int dim, bool bf16, void* out, int32_t* status, int num_sms, cudaStream_t stream);
+
 }  // namespace mpm

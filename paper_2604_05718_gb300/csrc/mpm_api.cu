@@ -285,6 +285,40 @@ mpm_status mpm_compose_gather(const void* merged, const int64_t* merged_offsets,
                                                 device_status, sms, static_cast<cudaStream_t>(stream)));
 }
 
+mpm_status mpm_pad_batch(const void* tokens, const int64_t* offsets, int32_t batch, int64_t rows, int32_t dim,
+                         mpm_dtype dtype, int64_t max_len, void* out, uint8_t* out_mask, int64_t* out_stats,
+                         int32_t* device_status, void* stream) {
+  if (!sizes_ok(rows, batch) || offsets == nullptr || max_len < 0) return MPM_ERR_INVALID_ARG;
+  mpm_status st = check_tokens(tokens, rows, dim, dtype);
+  if (st != MPM_OK) return st;
+  if (batch == 0) return MPM_OK;
+  if (max_len > 0 && (out == nullptr || !aligned16(out))) return out == nullptr ? MPM_ERR_INVALID_ARG : MPM_ERR_ALIGNMENT;
+  const size_t row_bytes = static_cast<size_t>(dim) * elem_size(dtype);
+  const int64_t out_rows = static_cast<int64_t>(batch) * max_len;
+  if (max_len > 0 && overlap(tokens, row_bytes * rows, out, row_bytes * out_rows)) return MPM_ERR_ALIASING;
+  const int sms = num_sms();
+  if (sms <= 0) return MPM_ERR_CUDA;
+  return cuda_status(mpm::launch_pad(tokens, offsets, batch, rows, max_len, dim, dtype == MPM_BF16, out, out_mask,
+                                     out_stats, device_status, sms, static_cast<cudaStream_t>(stream)));
+}
+
+mpm_status mpm_unpad_batch(const void* padded, int32_t batch, int64_t max_len, int32_t dim, mpm_dtype dtype,
+                           const int64_t* offsets, int64_t rows, void* out, int32_t* device_status, void* stream) {
+  if (!sizes_ok(rows, batch) || offsets == nullptr || max_len < 0) return MPM_ERR_INVALID_ARG;
+  const int64_t in_rows = static_cast<int64_t>(batch) * max_len;
+  mpm_status st = check_tokens(padded, in_rows, dim, dtype);
+  if (st != MPM_OK) return st;
+  if (rows == 0 || batch == 0) return MPM_OK;
+  if (out == nullptr) return MPM_ERR_INVALID_ARG;
+  if (!aligned16(out)) return MPM_ERR_ALIGNMENT;
+  const size_t row_bytes = static_cast<size_t>(dim) * elem_size(dtype);
+  if (overlap(padded, row_bytes * in_rows, out, row_bytes * rows)) return MPM_ERR_ALIASING;
+  const int sms = num_sms();
+  if (sms <= 0) return MPM_ERR_CUDA;
+  return cuda_status(mpm::launch_unpad(padded, batch, max_len, offsets, rows, dim, dtype == MPM_BF16, out,
+                                       device_status, sms, static_cast<cudaStream_t>(stream)));
+}
+
 mpm_status mpm_get_device_status(void* workspace, int32_t* host_code, void* stream) {
   if (workspace == nullptr || host_code == nullptr) return MPM_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);

@@ -28,7 +28,7 @@ STATUS_NAMES = {
 }
 EXPORTS = ("mpm_abi_version", "mpm_status_string", "mpm_merge_workspace_size", "mpm_merge", "mpm_merge_timed",
            "mpm_compose_maps", "mpm_unmerge_gather", "mpm_nearest_neighbors", "mpm_get_device_status",
-           "mpm_merge_no_alloc", "mpm_compose_gather")
+           "mpm_merge_no_alloc", "mpm_compose_gather", "mpm_pad_batch", "mpm_unpad_batch")
 
 _lib = None
 
@@ -57,6 +57,8 @@ def _declare(lib: ctypes.CDLL) -> None:
         "mpm_merge_no_alloc": (ctypes.c_int, [P, P, I32, I64, I32, ctypes.c_int, P, P, P, P]),
         "mpm_compose_gather": (ctypes.c_int, [P, P, I64, P, P, I64, P, P, I64, I32, I32, ctypes.c_int, P, P, P,
                                               P]),
+        "mpm_pad_batch": (ctypes.c_int, [P, P, I32, I64, I32, ctypes.c_int, I64, P, P, P, P, P]),
+        "mpm_unpad_batch": (ctypes.c_int, [P, I32, I64, I32, ctypes.c_int, P, I64, P, P, P]),
     }
     for name, (res, args) in sigs.items():
         fn = getattr(lib, name)
@@ -251,6 +253,49 @@ def compose_gather(merged: torch.Tensor, merged_offsets: torch.Tensor, map1: tor
                                             _dtype_code(merged), _ptr(out), _ptr(out_map),
                                             _ptr(device_status), _stream(dev))
     _check("mpm_compose_gather", code)
+    return out
+
+
+def pad_batch(tokens: torch.Tensor, offsets: torch.Tensor, max_len: int, out: torch.Tensor | None = None,
+              mask: torch.Tensor | None = None, stats: torch.Tensor | None = None,
+              device_status: torch.Tensor | None = None):
+    """Packed tokens -> ([B, max_len, D] padded, [B, max_len] uint8 key mask, int64 [3] N_b min/max/total).
+
+    Nothing is read back to the host: pass max_len = the largest N_b if the
+    caller knows it (e.g. from a host copy of offsets), or any upper bound.
+    """
+    _cuda(tokens, "tokens", ndim=2)
+    _cuda(offsets, "offsets", torch.int64, 1)
+    dev = tokens.device
+    batch = offsets.numel() - 1
+    max_len = int(max_len)
+    if out is None:
+        out = torch.empty(batch, max_len, tokens.shape[1], dtype=tokens.dtype, device=dev)
+    if mask is None:
+        mask = torch.empty(batch, max_len, dtype=torch.uint8, device=dev)
+    if stats is None:
+        stats = torch.empty(3, dtype=torch.int64, device=dev)
+    with torch.cuda.device(dev):
+        code = library().mpm_pad_batch(_ptr(tokens), _ptr(offsets), batch, tokens.shape[0], tokens.shape[1],
+                                       _dtype_code(tokens), max_len, _ptr(out), _ptr(mask), _ptr(stats),
+                                       _ptr(device_status), _stream(dev))
+    _check("mpm_pad_batch", code)
+    return out, mask, stats
+
+
+def unpad_batch(padded: torch.Tensor, offsets: torch.Tensor, rows: int | None = None,
+                out: torch.Tensor | None = None, device_status: torch.Tensor | None = None) -> torch.Tensor:
+    """[B, L, D] padded -> packed [rows, D] with out[offsets[b] + t] = padded[b, t]."""
+    _cuda(padded, "padded", ndim=3)
+    _cuda(offsets, "offsets", torch.int64, 1)
+    dev = padded.device
+    batch, max_len, dim = padded.shape
+    if out is None:
+        out = torch.empty(int(rows) if rows is not None else batch * max_len, dim, dtype=padded.dtype, device=dev)
+    with torch.cuda.device(dev):
+        code = library().mpm_unpad_batch(_ptr(padded), batch, max_len, dim, _dtype_code(padded), _ptr(offsets),
+                                         out.shape[0], _ptr(out), _ptr(device_status), _stream(dev))
+    _check("mpm_unpad_batch", code)
     return out
 
 

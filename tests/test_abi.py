@@ -124,4 +124,17 @@ def test_nn_compose_gather_validation(lib):
               P(FAKE * 4 + 8), None, None) == 8                                            # out_map overlaps map2
     assert cg(P(FAKE), P(FAKE), 10, P(FAKE), P(FAKE), 10, P(FAKE), P(FAKE), 10, 1, 60, 1, P(FAKE * 8), None,
               None, None) == 3                                                             # rows not 16-byte multiples
+    pad = lib.mpm_pad_batch
+    # (tokens, offsets, batch, rows, dim, dtype, max_len, out, out_mask, out_stats, device_status, stream)
+    assert pad(P(FAKE), None, 2, 10, 64, 1, 8, P(FAKE * 8), None, None, None, None) == 1         # no offsets
+    assert pad(P(FAKE), P(FAKE), 2, 10, 64, 1, -1, P(FAKE * 8), None, None, None, None) == 1     # negative L
+    assert pad(P(FAKE), P(FAKE), 2, 10, 64, 1, 8, None, None, None, None, None) == 1             # no output
+    assert pad(P(FAKE), P(FAKE), 2, 10, 64, 1, 8, P(FAKE + 128), None, None, None, None) == 8    # out overlaps tokens
+    assert pad(P(FAKE), P(FAKE), 2, 10, 64, 1, 8, P(FAKE * 8 + 4), None, None, None, None) == 3  # unaligned out
+    unpad = lib.mpm_unpad_batch
+    # (padded, batch, max_len, dim, dtype, offsets, rows, out, device_status, stream)
+    assert unpad(P(FAKE), 2, 8, 64, 1, None, 10, P(FAKE * 8), None, None) == 1                   # no offsets
+    assert unpad(P(FAKE), 2, 8, 64, 1, P(FAKE), 10, None, None, None) == 1                       # no output
+    assert unpad(P(FAKE), 2, 8, 64, 1, P(FAKE), 10, P(FAKE + 128), None, None) == 8              # out overlaps padded
+    assert unpad(P(FAKE), 2, 8, 60, 1, P(FAKE), 10, P(FAKE * 8), None, None) == 3                # 120-byte rows
     assert lib.mpm_get_device_status(None, None, None) == 1

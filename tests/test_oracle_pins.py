@@ -251,6 +251,32 @@ def test_batch_compose_gather_roundtrip():
         np.testing.assert_array_equal(up[a0:a1], z[m2.r[m1.out_offsets[b]:m1.out_offsets[b + 1]][m1.r[a0:a1]]])
 
 
+def test_pad_batch_hand():
+    # Three images of 2, 0 and 3 one-feature tokens, padded to L = 3 (values written out by hand).
+    x = np.array([[1.0], [2.0], [3.0], [4.0], [5.0]])
+    off = np.array([0, 2, 2, 5])
+    out, mask, stats = mpm_oracle.pad_batch(x, off, 3)
+    assert out[..., 0].tolist() == [[1, 2, 0], [0, 0, 0], [3, 4, 5]]
+    assert mask.tolist() == [[1, 1, 0], [0, 0, 0], [1, 1, 1]]
+    assert stats == (0, 3, 5)
+    # L = 2 cuts the third image to its first two rows.
+    out2, mask2, _ = mpm_oracle.pad_batch(x, off, 2)
+    assert out2[..., 0].tolist() == [[1, 2], [0, 0], [3, 4]]
+    assert mask2.tolist() == [[1, 1], [0, 0], [1, 1]]
+    assert mpm_oracle.unpad_batch(out, off)[:, 0].tolist() == [1, 2, 3, 4, 5]
+
+
+def test_pad_unpad_roundtrip_and_mask_counts():
+    batch = make_custom([7, 0, 1, 30, 12], 16, "f32", seed=4)
+    x = batch.tokens.double().numpy()
+    counts = np.diff(batch.offsets)
+    out, mask, stats = mpm_oracle.pad_batch(x, batch.offsets, int(counts.max()))
+    np.testing.assert_array_equal(mpm_oracle.unpad_batch(out, batch.offsets), x)
+    np.testing.assert_array_equal(mask.sum(axis=1), counts)
+    assert stats == (int(counts.min()), int(counts.max()), int(counts.sum()))
+    assert np.all(out[mask == 0] == 0)
+
+
 # ---------------------------------------------------------------------------
 # Second library: torch's cosine 1-NN (first-occurrence arg max, documented)
 # ---------------------------------------------------------------------------
