@@ -61,6 +61,7 @@ def parse_args():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=15.0, help="target CPU time of the oracle sample")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-chunked", action="store_true", help="skip the chunked-similarity measurement")
     return p.parse_args()
 
 
@@ -555,6 +556,40 @@ def run_mpm(args):
     padded["pad_frac"] = padded["pad_gbs"] / hbm_bw
     padded["unpad_frac"] = padded["unpad_gbs"] / hbm_bw
 
+    # ---------------- chunked similarity on the mixed-resolution workload ----------------
+    # One merge of the mixed workload (1024-4096 tokens per image) with the
+    # full similarity and with chunks of 1024 tokens (mpm_merge_chunked).
+    chunked = None
+    if rank == 0 and not args.no_chunked:
+        mcfg = CONFIGS["mixed"]
+        mb = make_batch(mcfg)
+        mx = mb.tokens.to(dev)
+        moff = torch.from_numpy(mb.offsets).to(dev)
+        mws = mpm.new_workspace(mb.rows, mcfg.batch, mcfg.dim, mx.dtype, dev)
+        mout = torch.empty_like(mx)
+        moo = torch.empty(mcfg.batch + 1, dtype=torch.int64, device=dev)
+        mmap = torch.empty(mb.rows, dtype=torch.int32, device=dev)
+        res = {}
+        for chunk in (0, 1024):
+            ts = []
+            for it in range(max(3, args.warmup) + 20):
+                flush.fill_(1)
+                flush_sum.copy_(flush.view(torch.int64).sum())
+                e = new_events(2)
+                e[0].record(stream)
+                mpm.merge(mx, moff, workspace=mws, out_tokens=mout, out_offsets=moo, out_map=mmap, chunk=chunk)
+                e[1].record(stream)
+                if it >= max(3, args.warmup):
+                    torch.cuda.synchronize(dev)
+                    ts.append(1e3 * e[0].elapsed_time(e[1]))
+            res[chunk] = (statistics.median(ts), int(moo[-1]))
+        chunked = {
+            "workload": mcfg.description, "tokens": mb.rows,
+            "merge_us_full": res[0][0], "merge_us_chunk_1024": res[1024][0],
+            "speedup": res[0][0] / res[1024][0],
+            "merged_tokens_full": res[0][1], "merged_tokens_chunk_1024": res[1024][1],
+        }
+
     # ---------------- end to end: host buffers, copies inside the timed region ----------------
     # A serving loop: every step copies its tokens and offsets in from pinned
     # host memory, runs the whole step (L2 flush, merge, stand-in noise,
@@ -639,6 +674,7 @@ def run_mpm(args):
             "roofline": roofline,
             "hbm_kernels": hbm_kernels,
             "padded_batch": padded,
+            "chunked_similarity": chunked,
             "kernels_us": kern,
             "ms_per_step_with_kernel_events": ms_with_kernel_events,
             "cpu_baseline": cpu_base,

@@ -167,6 +167,25 @@ MPM_API mpm_status mpm_merge_no_alloc(const void* tokens, const int64_t* offsets
                                       int64_t* out_offsets, int32_t* out_map, void* stream);
 
 /*
+ * Chunked similarity: mpm_merge with each token's nearest neighbour sought
+ * only among the `chunk` consecutive tokens (raster order) of its image that
+ * contain it (the last chunk of an image may be shorter).  The paper's
+ * discussion proposes chunking the similarity to bound the O(N^2) cosine pass
+ * at very large N (Section 5); the rest of Algorithm 1 is unchanged, so
+ * pairs never cross a chunk boundary.  A token alone in its chunk has no
+ * neighbour and stays a singleton.
+ *
+ *   chunk  0 = the whole image (exactly mpm_merge); otherwise a multiple of
+ *          256 (MPM_ERR_UNSUPPORTED if not; MPM_ERR_INVALID_ARG if negative).
+ * Every other argument is as for mpm_merge.  The cost of the affinity step
+ * drops from N_b^2 to about N_b * chunk per image.
+ */
+MPM_API mpm_status mpm_merge_chunked(const void* tokens, const int64_t* offsets, int32_t batch, int64_t rows,
+                                     int32_t dim, mpm_dtype dtype, int64_t chunk, void* out_tokens,
+                                     int64_t* out_offsets, int32_t* out_map, void* workspace,
+                                     size_t workspace_bytes, void* stream);
+
+/*
  * Map composition across two insertions (Eq. 3): r*(p) = r2(r1(p)).
  *
  *   map1      int32 [rows0]: stage-1 map, local to image b of offsets0
@@ -280,6 +299,16 @@ MPM_API mpm_status mpm_nearest_neighbors(const void* tokens, const int64_t* offs
                                  int64_t rows, int32_t dim, mpm_dtype dtype,
                                  mpm_nn_algo algo, int32_t* out_nn, float* out_score,
                                  void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * mpm_nearest_neighbors restricted to chunks, as in mpm_merge_chunked (test
+ * and diagnostics hook).  `algo` must be MPM_NN_AUTO, MPM_NN_TCGEN05_PAIR or
+ * MPM_NN_SIMT when chunk > 0; b(i) = -1 for a token alone in its chunk.
+ */
+MPM_API mpm_status mpm_nearest_neighbors_chunked(const void* tokens, const int64_t* offsets, int32_t batch,
+                                                 int64_t rows, int32_t dim, mpm_dtype dtype, mpm_nn_algo algo,
+                                                 int64_t chunk, int32_t* out_nn, float* out_score,
+                                                 void* workspace, size_t workspace_bytes, void* stream);
 
 /*
  * Copies the device status word of a merge workspace into *host_code

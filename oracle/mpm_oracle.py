@@ -63,11 +63,20 @@ def normalise_rows(x: np.ndarray) -> np.ndarray:
     return x / np.maximum(n, NORM_EPS)[:, None]
 
 
-def cosine_affinity(x: np.ndarray) -> np.ndarray:
-    """Eq. 1: S = X~ X~^T with the diagonal set to -inf (no self match)."""
+def cosine_affinity(x: np.ndarray, chunk: int | None = None) -> np.ndarray:
+    """Eq. 1: S = X~ X~^T with the diagonal set to -inf (no self match).
+
+    chunk: the chunked similarity that Section 5 proposes for very large N.
+    S_ij is kept only when i and j lie in the same run of `chunk`
+    consecutive tokens (raster order, the last run may be shorter); every
+    other entry is -inf.
+    """
     xt = normalise_rows(x)
     s = xt @ xt.T
     np.fill_diagonal(s, -np.inf)
+    if chunk:
+        run = np.arange(s.shape[0]) // int(chunk)
+        s[run[:, None] != run[None, :]] = -np.inf
     return s
 
 
@@ -96,11 +105,13 @@ class Neighbours:
         return ~(self.gap > NEAR_TIE_GAP)
 
 
-def nearest_neighbours(x: np.ndarray, affinity: np.ndarray | None = None) -> Neighbours:
+def nearest_neighbours(x: np.ndarray, affinity: np.ndarray | None = None,
+                       chunk: int | None = None) -> Neighbours:
     """Algorithm 1 step 3: b(i) = arg max_{j != i} S_ij.
 
     ``np.argmax`` returns the first maximal index, which is the lowest-j tie
-    rule.  For N == 1 the candidate set is empty and b(0) = -1.
+    rule.  For N == 1 the candidate set is empty and b(0) = -1; so is it for
+    a token alone in its chunk under the chunked similarity.
     """
     n = np.asarray(x).shape[0]
     if n == 0:
@@ -108,9 +119,10 @@ def nearest_neighbours(x: np.ndarray, affinity: np.ndarray | None = None) -> Nei
         return Neighbours(np.zeros(0, dtype=np.int64), e, e)
     if n == 1:
         return Neighbours(np.array([-1], dtype=np.int64), np.array([-np.inf]), np.array([-np.inf]))
-    s = cosine_affinity(x) if affinity is None else affinity
+    s = cosine_affinity(x, chunk) if affinity is None else affinity
     b = np.argmax(s, axis=1).astype(np.int64)
     top1 = s[np.arange(n), b]
+    b[np.isneginf(top1)] = -1  # no candidate at all
     if n == 2:
         top2 = np.full(n, -np.inf)
     else:
@@ -201,10 +213,10 @@ class MergeResult:
         return int(np.sum(self.rep_partner >= 0))
 
 
-def merge_image(x: np.ndarray) -> MergeResult:
-    """Algorithm 1 on a single image's tokens X (N x d)."""
+def merge_image(x: np.ndarray, chunk: int | None = None) -> MergeResult:
+    """Algorithm 1 on a single image's tokens X (N x d); chunk as in cosine_affinity."""
     x = np.asarray(x, dtype=np.float64)
-    nn = nearest_neighbours(x)
+    nn = nearest_neighbours(x, chunk=chunk)
     partner = mutual_partners(nn.b)
     r, rep_index, rep_partner = compact_map(partner)
     x_out = cluster_average(x, r, int(rep_index.shape[0]))
@@ -239,15 +251,15 @@ class BatchMerge:
     images: list             # list[MergeResult]
 
 
-def merge_batch(tokens: np.ndarray, offsets: np.ndarray) -> BatchMerge:
-    """Algorithm 1 applied to each image of a packed batch."""
+def merge_batch(tokens: np.ndarray, offsets: np.ndarray, chunk: int | None = None) -> BatchMerge:
+    """Algorithm 1 applied to each image of a packed batch (chunk as in cosine_affinity)."""
     tokens = np.asarray(tokens, dtype=np.float64)
     offsets = np.asarray(offsets, dtype=np.int64)
     b_count = offsets.shape[0] - 1
     outs, maps, images = [], [], []
     out_offsets = np.zeros(b_count + 1, dtype=np.int64)
     for b in range(b_count):
-        res = merge_image(tokens[offsets[b]:offsets[b + 1]])
+        res = merge_image(tokens[offsets[b]:offsets[b + 1]], chunk)
         images.append(res)
         outs.append(res.x_out)
         maps.append(res.r)

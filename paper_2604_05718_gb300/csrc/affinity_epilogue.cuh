@@ -110,14 +110,15 @@ __device__ __forceinline__ void epilogue_piece(const uint32_t (&v)[16], const fl
 }
 
 // Column candidate of tile column c + lane from the scratch entries of the
-// 32 columns c .. c + 31 (0 when there is none).
+// 32 columns c .. c + 31 (0 when there is none).  `origin` is added to the
+// winning row for the key: the tile's first token within its image.
 __device__ __forceinline__ unsigned long long column_candidate(const uint2* scratch, int lane, int row_base, int n,
-                                                               int col) {
+                                                               int col, int origin) {
   __syncwarp();
   const uint2 r = scratch[lane];
   __syncwarp();
   const int winner = row_base + __ffs(static_cast<int>(r.y)) - 1;
-  return (r.y != 0u && winner < n && col < n) ? make_key(__uint_as_float(r.x), winner) : 0ull;
+  return (r.y != 0u && winner < n && col < n) ? make_key(__uint_as_float(r.x), origin + winner) : 0ull;
 }
 
 // A warp's whole COLS-column slice of one accumulator (TMEM columns
@@ -130,7 +131,8 @@ __device__ __forceinline__ unsigned long long column_candidate(const uint2* scra
 template <int COLS, bool DIAG, bool COL>
 __device__ __forceinline__ void epilogue_slice(uint32_t taddr, const float* sc, int c0, int jd, float& best,
                                                int& bj, float inv_i, int lane, int row_base, int n, int col0,
-                                               uint2* scratch, unsigned long long (&colcand)[COLS / 32]) {
+                                               int origin, uint2* scratch,
+                                               unsigned long long (&colcand)[COLS / 32]) {
   static_assert(COLS % 32 == 0, "slices are whole 32-column pairs of pieces");
   float best0 = -INFINITY, best1 = -INFINITY;
   int bj0 = -1, bj1 = -1;
@@ -146,7 +148,7 @@ __device__ __forceinline__ void epilogue_slice(uint32_t taddr, const float* sc, 
     if (h + 1 < COLS / 32) ptx::tmem_ld_32x32b_x16(taddr + 32 * h + 32, va);
     epilogue_piece<DIAG, COL>(vb, sc, c + 16, jd, best0, bj0, best1, bj1, inv_i, lane, scratch, 16);
     if (COL) {
-      const unsigned long long key = column_candidate(scratch, lane, row_base, n, col0 + c + lane);
+      const unsigned long long key = column_candidate(scratch, lane, row_base, n, col0 + c + lane, origin);
 #pragma unroll
       for (int g = 0; g < COLS / 32; ++g)
         if (g == h) colcand[g] = key;

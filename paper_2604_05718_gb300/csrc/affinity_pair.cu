@@ -77,21 +77,23 @@ struct Control {
 };
 
 struct Item {
-  int64_t base;
-  int n;
-  int row0;  // first local row of the tile (a multiple of 256)
-  int col0;  // first local column of the tile (a multiple of 256)
+  int64_t base;  // global row of the first token of the tile's chunk
+  int n;         // tokens in the chunk (the image without chunking)
+  int row0;      // first row of the tile within the chunk (a multiple of 256)
+  int col0;      // first column of the tile within the chunk (a multiple of 256)
+  int origin;    // index of the chunk's first token within its image
 };
 
 constexpr size_t SMEM_BYTES = 1024 + static_cast<size_t>(STAGES) * STAGE_BYTES + EPI_WARPS * EPI_COLS * sizeof(float) +
                               sizeof(Control) + 16 + kMaxItems * sizeof(Item) +
                               2 * (kMaxStagedImages + 1) * sizeof(int64_t) + EPI_WARPS * 32 * sizeof(uint2);
 
-// Item w of the launch: image by the plan, then the upper-triangle tile (I, J),
-// J >= I, numbered row by row: row I starts at P(I) = I R - I (I - 1) / 2.
-// `plan` and `soff` are the work plan and sanitised offsets, in shared or
-// global memory.
-__device__ __forceinline__ Item decode_pair_item(const int64_t* plan, const int64_t* soff, int batch, int64_t w) {
+// Item w of the launch: image by the plan, its chunk, then the
+// upper-triangle tile (I, J), J >= I, of that chunk numbered row by row: row
+// I starts at P(I) = I R - I (I - 1) / 2.  `plan` and `soff` are the work
+// plan and sanitised offsets, in shared or global memory.
+__device__ __forceinline__ Item decode_pair_item(const int64_t* plan, const int64_t* soff, int batch, int64_t w,
+                                                 int64_t chunk) {
   int lo_b = 0, hi_b = batch - 1;
   while (lo_b < hi_b) {
     const int mid = (lo_b + hi_b + 1) >> 1;
@@ -99,9 +101,12 @@ __device__ __forceinline__ Item decode_pair_item(const int64_t* plan, const int6
   }
   const int b = lo_b;
   int64_t local = w - plan[b];
+  const ChunkItem ch = locate_chunk(local, soff[b + 1] - soff[b], AffinityTile{TILE, TILE, AffinityTile::kUpperSquare, chunk});
+  local = ch.local;
   Item it;
-  it.base = soff[b];
-  it.n = static_cast<int>(soff[b + 1] - it.base);
+  it.base = soff[b] + ch.start;
+  it.n = static_cast<int>(ch.len);
+  it.origin = static_cast<int>(ch.start);
   const int64_t r = (it.n + TILE - 1) / TILE;
   int64_t lo = 0, hi = r - 1;
   while (lo < hi) {
@@ -220,7 +225,7 @@ __device__ __forceinline__ void fail(Control* ctl, int32_t* status, int32_t role
 }
 
 __global__ void __launch_bounds__(THREADS, 1)
-    affinity_pair_kernel(const __grid_constant__ CUtensorMap tmap, int batch, int dim, Workspace ws) {
+    affinity_pair_kernel(const __grid_constant__ CUtensorMap tmap, int batch, int dim, int64_t chunk, Workspace ws) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024u - (ptx::smem_addr(smem_raw) & 1023u)) & 1023u);
   uint8_t* stages = smem;
@@ -283,10 +288,10 @@ __global__ void __launch_bounds__(THREADS, 1)
   const int64_t total = plan[batch];
   const int64_t count = total > cid ? (total - 1 - cid) / clusters + 1 : 0;
   for (int64_t k = threadIdx.x; k < count && k < kMaxItems; k += THREADS)
-    items[k] = decode_pair_item(plan, soff, batch, cid + k * clusters);
+    items[k] = decode_pair_item(plan, soff, batch, cid + k * clusters, chunk);
   __syncthreads();
   auto item = [&](int64_t k) -> Item {
-    return k < kMaxItems ? items[k] : decode_pair_item(plan, soff, batch, cid + k * clusters);
+    return k < kMaxItems ? items[k] : decode_pair_item(plan, soff, batch, cid + k * clusters, chunk);
   };
   volatile int* abort_flag = &ctl->abort_flag;
 
@@ -437,11 +442,11 @@ __global__ void __launch_bounds__(THREADS, 1)
       for (int h = 0; h < EPI_COLS / 32; ++h) colcand[h] = 0ull;
       const uint32_t taddr = tmem + lane_addr + static_cast<uint32_t>(acc * TILE + c0);
       if (diag) {
-        epilogue_slice<EPI_COLS, true, false>(taddr, sc, c0, jd, best, bj, inv_i, lane, row_base, it.n, it.col0, scr,
-                                              colcand);
+        epilogue_slice<EPI_COLS, true, false>(taddr, sc, c0, jd, best, bj, inv_i, lane, row_base, it.n, it.col0,
+                                              it.origin, scr, colcand);
       } else if (col_update) {
-        epilogue_slice<EPI_COLS, false, true>(taddr, sc, c0, jd, best, bj, inv_i, lane, row_base, it.n, it.col0, scr,
-                                              colcand);
+        epilogue_slice<EPI_COLS, false, true>(taddr, sc, c0, jd, best, bj, inv_i, lane, row_base, it.n, it.col0,
+                                              it.origin, scr, colcand);
       }
       // Release the accumulator first, then merge this tile's candidates.
       ptx::tc_fence_before_sync();
@@ -451,7 +456,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         __syncwarp();
         if (lane == 0) remote_arrive(acc == 0 ? empty_leader0 : empty_leader1);
       }
-      if (bj >= 0 && row < it.n) atomicMax(ws.keys + it.base + row, make_key(best, it.col0 + bj));
+      if (bj >= 0 && row < it.n) atomicMax(ws.keys + it.base + row, make_key(best, it.origin + it.col0 + bj));
 #pragma unroll
       for (int h = 0; h < EPI_COLS / 32; ++h)
         if (colcand[h] != 0ull) atomicMax(ws.keys + it.base + it.col0 + c0 + 32 * h + lane, colcand[h]);
@@ -488,8 +493,8 @@ PFN_cuTensorMapEncodeTiled_v12000 encoder() {
 
 AffinityTile pair_tile() { return {TILE, TILE, AffinityTile::kUpperSquare}; }
 
-cudaError_t launch_affinity_pair(const void* tokens, int batch, int64_t rows, int dim, const Workspace& ws,
-                                 int num_sms, cudaStream_t stream) {
+cudaError_t launch_affinity_pair(const void* tokens, int batch, int64_t rows, int dim, int64_t chunk,
+                                 const Workspace& ws, int num_sms, cudaStream_t stream) {
   PFN_cuTensorMapEncodeTiled_v12000 encode = encoder();
   if (encode == nullptr) return cudaErrorNotSupported;
   CUtensorMap map;
@@ -527,7 +532,7 @@ cudaError_t launch_affinity_pair(const void* tokens, int batch, int64_t rows, in
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, affinity_pair_kernel, map, batch, dim, ws);
+  return cudaLaunchKernelEx(&cfg, affinity_pair_kernel, map, batch, dim, chunk, ws);
 }
 
 }  // namespace mpm

@@ -22,7 +22,7 @@ __device__ __forceinline__ float load_elem(const uint8_t* tokens, int64_t row, i
 
 template <bool BF16>
 __global__ void __launch_bounds__(kThreads) affinity_simt_kernel(const uint8_t* __restrict__ tokens, int batch,
-                                                                 int dim, Workspace ws) {
+                                                                 int dim, int64_t chunk, Workspace ws) {
   wait_for_previous_grid();
   __shared__ __align__(16) float As[BK][BM + 4];
   __shared__ __align__(16) float Bs[BK][BN + 4];
@@ -32,9 +32,14 @@ __global__ void __launch_bounds__(kThreads) affinity_simt_kernel(const uint8_t* 
   const int64_t total = ws.plan[batch];
   for (int64_t w = blockIdx.x; w < total; w += gridDim.x) {
     const int b = find_item_image(ws.plan, batch, w);
-    const int64_t local = w - ws.plan[b];
-    const int64_t base = ws.soff[b];
-    const int n = static_cast<int>(ws.soff[b + 1] - base);
+    // Tiles of the item's chunk (the whole image without chunking); keys
+    // hold indices within the image, so chunk-relative columns get `origin`.
+    const ChunkItem ch = locate_chunk(w - ws.plan[b], ws.soff[b + 1] - ws.soff[b],
+                                      AffinityTile{BM, BN, AffinityTile::kDense, chunk});
+    const int64_t local = ch.local;
+    const int64_t base = ws.soff[b] + ch.start;
+    const int n = static_cast<int>(ch.len);
+    const int origin = static_cast<int>(ch.start);
     const int ct = (n + BN - 1) / BN;
     const int r0 = static_cast<int>(local / ct) * BM;
     const int c0 = static_cast<int>(local % ct) * BN;
@@ -87,7 +92,7 @@ __global__ void __launch_bounds__(kThreads) affinity_simt_kernel(const uint8_t* 
           bj = c0 + col;
         }
       }
-      unsigned long long key = bj >= 0 ? make_key(best, bj) : 0ull;
+      unsigned long long key = bj >= 0 ? make_key(best, origin + bj) : 0ull;
 #pragma unroll
       for (int d = 8; d > 0; d >>= 1) {
         const unsigned long long o = __shfl_xor_sync(0xFFFFFFFFu, key, d);
@@ -103,12 +108,15 @@ __global__ void __launch_bounds__(kThreads) affinity_simt_kernel(const uint8_t* 
 
 AffinityTile simt_tile() { return {BM, BN, AffinityTile::kDense}; }
 
-cudaError_t launch_affinity_simt(const void* tokens, int batch, int dim, bool bf16, const Workspace& ws,
-                                 int num_sms, cudaStream_t stream) {
+cudaError_t launch_affinity_simt(const void* tokens, int batch, int dim, bool bf16, int64_t chunk,
+                                 const Workspace& ws, int num_sms, cudaStream_t stream) {
   const int grid = (num_sms > 0 ? num_sms : 1) * 4;
   const uint8_t* t = static_cast<const uint8_t*>(tokens);
-  if (bf16) return launch_dependent(affinity_simt_kernel<true>, dim3(grid), dim3(kThreads), 0, stream, t, batch, dim, ws);
-  return launch_dependent(affinity_simt_kernel<false>, dim3(grid), dim3(kThreads), 0, stream, t, batch, dim, ws);
+  if (bf16)
+    return launch_dependent(affinity_simt_kernel<true>, dim3(grid), dim3(kThreads), 0, stream, t, batch, dim, chunk,
+                            ws);
+  return launch_dependent(affinity_simt_kernel<false>, dim3(grid), dim3(kThreads), 0, stream, t, batch, dim, chunk,
+                          ws);
 }
 
 }  // namespace mpm

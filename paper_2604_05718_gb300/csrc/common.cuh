@@ -75,6 +75,29 @@ __host__ __device__ __forceinline__ int64_t affinity_tiles(int64_t n, int rows, 
   return 2 * q * c - q * (q - 1) + (r & 1) * (c - q);
 }
 
+// Work items of an image of n tokens: the tiles of every chunk (the whole
+// image when t.chunk == 0; the last chunk may be shorter).
+__host__ __device__ __forceinline__ int64_t image_items(int64_t n, const AffinityTile& t) {
+  if (t.chunk <= 0 || n <= t.chunk) return affinity_tiles(n, t.rows, t.cols, t.mode);
+  const int64_t full = n / t.chunk, last = n - full * t.chunk;
+  return full * affinity_tiles(t.chunk, t.rows, t.cols, t.mode) +
+         (last > 0 ? affinity_tiles(last, t.rows, t.cols, t.mode) : 0);
+}
+
+// The chunk of work item `local` of an image of n tokens: its first token,
+// its length and the item's index within it.
+struct ChunkItem {
+  int64_t start, len, local;
+};
+__device__ __forceinline__ ChunkItem locate_chunk(int64_t local, int64_t n, const AffinityTile& t) {
+  if (t.chunk <= 0 || n <= t.chunk) return {0, n, local};
+  const int64_t per = affinity_tiles(t.chunk, t.rows, t.cols, t.mode);
+  const int64_t full = n / t.chunk;
+  const int64_t c = local / per;
+  if (c < full) return {c * t.chunk, t.chunk, local - c * per};
+  return {full * t.chunk, n - full * t.chunk, local - full * per};
+}
+
 // A total order on floats as unsigned integers (larger float -> larger key).
 __device__ __forceinline__ uint32_t order_f32(float f) {
   uint32_t u = __float_as_uint(f);

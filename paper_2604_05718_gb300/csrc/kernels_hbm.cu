@@ -85,7 +85,7 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(const uint8_t* __restric
       int64_t items = 0;
       if (idx < batch) {
         const int64_t n = ws.soff[idx + 1] - ws.soff[idx];
-        items = affinity_tiles(n, tile.rows, tile.cols, tile.mode);
+        items = image_items(n, tile);
       }
       int64_t total;
       const int64_t incl = block_incl_sum<int64_t>(items, sh, &total);
@@ -143,7 +143,7 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(const uint8_t* __restric
 // ---------------------------------------------------------------------------
 constexpr int kScanThreads = 1024;
 
-__global__ void __launch_bounds__(kScanThreads) mutual_compact_kernel(int batch, Workspace ws,
+__global__ void __launch_bounds__(kScanThreads) mutual_compact_kernel(int batch, int64_t chunk, Workspace ws,
                                                                       int32_t* __restrict__ out_map,
                                                                       int64_t* __restrict__ out_offsets) {
   wait_for_previous_grid();
@@ -159,7 +159,11 @@ __global__ void __launch_bounds__(kScanThreads) mutual_compact_kernel(int batch,
     int rep = 0, partner = -1;
     if (i < n) {
       int j = key_index(ws.keys[base + i]);
-      if (j >= n || j == i || (j < 0 && n > 1)) {
+      // b(i) lies in i's chunk (the whole image without chunking), and only a
+      // token alone in its chunk has none.
+      const int64_t cstart = chunk > 0 ? (i / chunk) * chunk : 0;
+      const int64_t clen = chunk > 0 ? (n - cstart < chunk ? n - cstart : chunk) : n;
+      if (j >= n || j == i || (j < 0 && clen > 1) || (j >= 0 && (j < cstart || j >= cstart + clen))) {
         report(ws.status, MPM_ERR_DEVICE_CHECK, static_cast<int32_t>(base + i));
         j = -1;
       }
@@ -390,10 +394,10 @@ cudaError_t launch_prep(const void* tokens, const int64_t* offsets, int batch, i
                           static_cast<const uint8_t*>(tokens), offsets, batch, rows, row_bytes, bf16, tile, ws);
 }
 
-cudaError_t launch_mutual_compact(int batch, const Workspace& ws, int32_t* out_map,
+cudaError_t launch_mutual_compact(int batch, int64_t chunk, const Workspace& ws, int32_t* out_map,
                                   int64_t* out_offsets, cudaStream_t stream) {
-  return launch_dependent(mutual_compact_kernel, dim3(batch), dim3(kScanThreads), 0, stream, batch, ws, out_map,
-                          out_offsets);
+  return launch_dependent(mutual_compact_kernel, dim3(batch), dim3(kScanThreads), 0, stream, batch, chunk, ws,
+                          out_map, out_offsets);
 }
 
 cudaError_t launch_pair_average(const void* tokens, void* out_tokens, int batch, int64_t rows,

@@ -33,6 +33,9 @@ struct AffinityTile {
   int rows;
   int cols;
   int mode;
+  // Chunked similarity: tokens are compared only within runs of `chunk`
+  // consecutive tokens of their image (0 = the whole image).
+  int64_t chunk = 0;
 };
 
 // Inverse row norms, key reset, offsets sanitisation and the work plan.
@@ -41,7 +44,7 @@ cudaError_t launch_prep(const void* tokens, const int64_t* offsets, int batch, i
                         cudaStream_t stream);
 
 // CUDA-core affinity + arg max (any dtype).
-cudaError_t launch_affinity_simt(const void* tokens, int batch, int dim, bool bf16,
+cudaError_t launch_affinity_simt(const void* tokens, int batch, int dim, bool bf16, int64_t chunk,
                                  const Workspace& ws, int num_sms, cudaStream_t stream);
 AffinityTile simt_tile();
 
@@ -52,12 +55,12 @@ AffinityTile tc_tile(bool symmetric);
 bool tc_available();
 
 // Symmetric affinity + arg max on SM pairs (tcgen05.mma.cta_group::2, bf16).
-cudaError_t launch_affinity_pair(const void* tokens, int batch, int64_t rows, int dim, const Workspace& ws,
-                                 int num_sms, cudaStream_t stream);
+cudaError_t launch_affinity_pair(const void* tokens, int batch, int64_t rows, int dim, int64_t chunk,
+                                 const Workspace& ws, int num_sms, cudaStream_t stream);
 AffinityTile pair_tile();
 
 // Mutual check, representative scan, per-image counts, output offsets.
-cudaError_t launch_mutual_compact(int batch, const Workspace& ws, int32_t* out_map,
+cudaError_t launch_mutual_compact(int batch, int64_t chunk, const Workspace& ws, int32_t* out_map,
                                   int64_t* out_offsets, cudaStream_t stream);
 
 // Pair average + compaction into the packed output.

@@ -14,6 +14,8 @@ namespace {
 using mpm::Workspace;
 
 constexpr size_t kAlign = 256;
+// Chunks of the chunked similarity are whole tiles of the SM-pair kernel.
+constexpr int64_t kChunkQuantum = 256;
 
 size_t round_up(size_t v) { return (v + kAlign - 1) / kAlign * kAlign; }
 
@@ -103,35 +105,113 @@ bool is_tensor_core(mpm_nn_algo a) {
   return a == MPM_NN_TCGEN05 || a == MPM_NN_TCGEN05_SYM || a == MPM_NN_TCGEN05_PAIR;
 }
 
-mpm::AffinityTile tile_of(mpm_nn_algo a) {
-  if (a == MPM_NN_TCGEN05_PAIR) return mpm::pair_tile();
-  if (a == MPM_NN_TCGEN05 || a == MPM_NN_TCGEN05_SYM) return mpm::tc_tile(a == MPM_NN_TCGEN05_SYM);
-  return mpm::simt_tile();
+mpm::AffinityTile tile_of(mpm_nn_algo a, int64_t chunk) {
+  mpm::AffinityTile t = a == MPM_NN_TCGEN05_PAIR                              ? mpm::pair_tile()
+                        : (a == MPM_NN_TCGEN05 || a == MPM_NN_TCGEN05_SYM) ? mpm::tc_tile(a == MPM_NN_TCGEN05_SYM)
+                                                                            : mpm::simt_tile();
+  t.chunk = chunk;
+  return t;
+}
+
+// Chunked similarity runs on the SM-pair tensor-core kernel and the fp32
+// kernel, with chunks of whole 256-token tiles.
+mpm_status check_chunk(mpm_nn_algo algo, int64_t chunk) {
+  if (chunk < 0) return MPM_ERR_INVALID_ARG;
+  if (chunk == 0) return MPM_OK;
+  if (chunk % kChunkQuantum != 0) return MPM_ERR_UNSUPPORTED;
+  if (algo != MPM_NN_TCGEN05_PAIR && algo != MPM_NN_SIMT) return MPM_ERR_UNSUPPORTED;
+  return MPM_OK;
 }
 
 cudaError_t launch_affinity(mpm_nn_algo a, const void* tokens, int batch, int64_t rows, int dim, bool bf16,
-                            const Workspace& ws, int sms, cudaStream_t s) {
-  if (a == MPM_NN_TCGEN05_PAIR) return mpm::launch_affinity_pair(tokens, batch, rows, dim, ws, sms, s);
+                            int64_t chunk, const Workspace& ws, int sms, cudaStream_t s) {
+  if (a == MPM_NN_TCGEN05_PAIR) return mpm::launch_affinity_pair(tokens, batch, rows, dim, chunk, ws, sms, s);
   if (a == MPM_NN_TCGEN05 || a == MPM_NN_TCGEN05_SYM)
     return mpm::launch_affinity_tc(tokens, batch, rows, dim, a == MPM_NN_TCGEN05_SYM, ws, sms, s);
-  return mpm::launch_affinity_simt(tokens, batch, dim, bf16, ws, sms, s);
+  return mpm::launch_affinity_simt(tokens, batch, dim, bf16, chunk, ws, sms, s);
 }
 
-// The affinity + arg max stage shared by mpm_merge and mpm_nearest_neighbors.
+// The affinity + arg max stage shared by the merge and nearest-neighbour
+// entry points.
 mpm_status run_affinity(const void* tokens, const int64_t* offsets, int32_t batch, int64_t rows, int32_t dim,
-                        mpm_dtype dtype, mpm_nn_algo algo, const Workspace& ws, cudaStream_t stream) {
+                        mpm_dtype dtype, mpm_nn_algo algo, int64_t chunk, const Workspace& ws,
+                        cudaStream_t stream) {
   const bool bf16 = dtype == MPM_BF16;
   if (algo == MPM_NN_AUTO) algo = default_algo(dtype);
   const bool tc = is_tensor_core(algo);
   if (algo != MPM_NN_SIMT && !tc) return MPM_ERR_INVALID_ARG;
   if (tc && !bf16) return MPM_ERR_UNSUPPORTED;
+  const mpm_status cs = check_chunk(algo, chunk);
+  if (cs != MPM_OK) return cs;
   if (tc && !mpm::tc_available()) return MPM_ERR_UNSUPPORTED;
   const int sms = num_sms();
   if (sms <= 0) return MPM_ERR_CUDA;
-  cudaError_t e = mpm::launch_prep(tokens, offsets, batch, rows, dim, bf16, tile_of(algo), ws, sms, stream);
+  cudaError_t e = mpm::launch_prep(tokens, offsets, batch, rows, dim, bf16, tile_of(algo, chunk), ws, sms, stream);
   if (e != cudaSuccess) return MPM_ERR_CUDA;
   if (rows == 0) return MPM_OK;  // every image is empty: nothing to compare
-  return cuda_status(launch_affinity(algo, tokens, batch, rows, dim, bf16, ws, sms, stream));
+  return cuda_status(launch_affinity(algo, tokens, batch, rows, dim, bf16, chunk, ws, sms, stream));
+}
+
+mpm_status nearest_neighbors_impl(const void* tokens, const int64_t* offsets, int32_t batch, int64_t rows,
+                                  int32_t dim, mpm_dtype dtype, mpm_nn_algo algo, int64_t chunk, int32_t* out_nn,
+                                  float* out_score, void* workspace, size_t workspace_bytes, void* stream) {
+  if (!sizes_ok(rows, batch) || offsets == nullptr || out_nn == nullptr) return MPM_ERR_INVALID_ARG;
+  mpm_status st = check_tokens(tokens, rows, dim, dtype);
+  if (st != MPM_OK) return st;
+  if (workspace == nullptr || (reinterpret_cast<uintptr_t>(workspace) % kAlign) != 0 ||
+      workspace_bytes < layout(rows, batch).total)
+    return MPM_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const Workspace ws = carve(workspace, rows, batch);
+  st = run_affinity(tokens, offsets, batch, rows, dim, dtype, algo, chunk, ws, s);
+  if (st != MPM_OK) return st;
+  return cuda_status(mpm::launch_decode_nn(batch, rows, ws, out_nn, out_score, num_sms(), s));
+}
+
+mpm_status merge_impl(const void* tokens, const int64_t* offsets, int32_t batch, int64_t rows, int32_t dim,
+                      mpm_dtype dtype, int64_t chunk, void* out_tokens, int64_t* out_offsets, int32_t* out_map,
+                      void* workspace, size_t workspace_bytes, void* stream, void* const* stage_events) {
+  if (!sizes_ok(rows, batch) || offsets == nullptr || out_offsets == nullptr) return MPM_ERR_INVALID_ARG;
+  if (rows > 0 && (out_tokens == nullptr || out_map == nullptr)) return MPM_ERR_INVALID_ARG;
+  mpm_status st = check_tokens(tokens, rows, dim, dtype);
+  if (st != MPM_OK) return st;
+  if (!aligned16(out_tokens)) return MPM_ERR_ALIGNMENT;
+  const size_t bytes = static_cast<size_t>(rows) * dim * elem_size(dtype);
+  if (overlap(tokens, bytes, out_tokens, bytes)) return MPM_ERR_ALIASING;
+  if (workspace == nullptr || (reinterpret_cast<uintptr_t>(workspace) % kAlign) != 0 ||
+      workspace_bytes < layout(rows, batch).total)
+    return MPM_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const Workspace ws = carve(workspace, rows, batch);
+  const bool bf16 = dtype == MPM_BF16;
+  const mpm_nn_algo algo = default_algo(dtype);
+  st = check_chunk(algo, chunk);
+  if (st != MPM_OK) return st;
+  if (is_tensor_core(algo) && !mpm::tc_available()) return MPM_ERR_UNSUPPORTED;
+  const int sms = num_sms();
+  if (sms <= 0) return MPM_ERR_CUDA;
+  // Records stage_events[idx] (if profiling) on the launch stream.
+  auto mark = [&](int idx) -> bool {
+    if (stage_events == nullptr) return true;
+    return cudaEventRecord(static_cast<cudaEvent_t>(stage_events[idx]), s) == cudaSuccess;
+  };
+  const mpm::AffinityTile tile = tile_of(algo, chunk);
+  cudaError_t e = cudaSuccess;
+  if (!mark(0)) return MPM_ERR_CUDA;
+  e = mpm::launch_prep(tokens, offsets, batch, rows, dim, bf16, tile, ws, sms, s);
+  if (e != cudaSuccess || !mark(1) || !mark(2)) return MPM_ERR_CUDA;
+  if (rows > 0) {
+    e = launch_affinity(algo, tokens, batch, rows, dim, bf16, chunk, ws, sms, s);
+    if (e != cudaSuccess) return MPM_ERR_CUDA;
+  }
+  if (!mark(3) || !mark(4)) return MPM_ERR_CUDA;
+  e = mpm::launch_mutual_compact(batch, chunk, ws, out_map, out_offsets, s);
+  if (e != cudaSuccess || !mark(5) || !mark(6)) return MPM_ERR_CUDA;
+  if (rows > 0) {
+    e = mpm::launch_pair_average(tokens, out_tokens, batch, rows, dim, bf16, ws, out_offsets, sms, s);
+    if (e != cudaSuccess) return MPM_ERR_CUDA;
+  }
+  return mark(7) ? MPM_OK : MPM_ERR_CUDA;
 }
 
 }  // namespace
@@ -163,69 +243,38 @@ size_t mpm_merge_workspace_size(int64_t rows, int32_t batch, int32_t dim, mpm_dt
 mpm_status mpm_nearest_neighbors(const void* tokens, const int64_t* offsets, int32_t batch, int64_t rows,
                                  int32_t dim, mpm_dtype dtype, mpm_nn_algo algo, int32_t* out_nn,
                                  float* out_score, void* workspace, size_t workspace_bytes, void* stream) {
-  if (!sizes_ok(rows, batch) || offsets == nullptr || out_nn == nullptr) return MPM_ERR_INVALID_ARG;
-  mpm_status st = check_tokens(tokens, rows, dim, dtype);
-  if (st != MPM_OK) return st;
-  if (workspace == nullptr || (reinterpret_cast<uintptr_t>(workspace) % kAlign) != 0 ||
-      workspace_bytes < layout(rows, batch).total)
-    return MPM_ERR_WORKSPACE;
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const Workspace ws = carve(workspace, rows, batch);
-  st = run_affinity(tokens, offsets, batch, rows, dim, dtype, algo, ws, s);
-  if (st != MPM_OK) return st;
-  return cuda_status(mpm::launch_decode_nn(batch, rows, ws, out_nn, out_score, num_sms(), s));
+  return nearest_neighbors_impl(tokens, offsets, batch, rows, dim, dtype, algo, 0, out_nn, out_score, workspace,
+                                workspace_bytes, stream);
+}
+
+mpm_status mpm_nearest_neighbors_chunked(const void* tokens, const int64_t* offsets, int32_t batch, int64_t rows,
+                                         int32_t dim, mpm_dtype dtype, mpm_nn_algo algo, int64_t chunk,
+                                         int32_t* out_nn, float* out_score, void* workspace,
+                                         size_t workspace_bytes, void* stream) {
+  return nearest_neighbors_impl(tokens, offsets, batch, rows, dim, dtype, algo, chunk, out_nn, out_score,
+                                workspace, workspace_bytes, stream);
 }
 
 mpm_status mpm_merge_timed(const void* tokens, const int64_t* offsets, int32_t batch, int64_t rows,
                            int32_t dim, mpm_dtype dtype, void* out_tokens, int64_t* out_offsets,
                            int32_t* out_map, void* workspace, size_t workspace_bytes, void* stream,
                            void* const* stage_events) {
-  if (!sizes_ok(rows, batch) || offsets == nullptr || out_offsets == nullptr) return MPM_ERR_INVALID_ARG;
-  if (rows > 0 && (out_tokens == nullptr || out_map == nullptr)) return MPM_ERR_INVALID_ARG;
-  mpm_status st = check_tokens(tokens, rows, dim, dtype);
-  if (st != MPM_OK) return st;
-  if (!aligned16(out_tokens)) return MPM_ERR_ALIGNMENT;
-  const size_t bytes = static_cast<size_t>(rows) * dim * elem_size(dtype);
-  if (overlap(tokens, bytes, out_tokens, bytes)) return MPM_ERR_ALIASING;
-  if (workspace == nullptr || (reinterpret_cast<uintptr_t>(workspace) % kAlign) != 0 ||
-      workspace_bytes < layout(rows, batch).total)
-    return MPM_ERR_WORKSPACE;
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const Workspace ws = carve(workspace, rows, batch);
-  const bool bf16 = dtype == MPM_BF16;
-  const mpm_nn_algo algo = default_algo(dtype);
-  if (is_tensor_core(algo) && !mpm::tc_available()) return MPM_ERR_UNSUPPORTED;
-  const int sms = num_sms();
-  if (sms <= 0) return MPM_ERR_CUDA;
-  // Records stage_events[idx] (if profiling) on the launch stream.
-  auto mark = [&](int idx) -> bool {
-    if (stage_events == nullptr) return true;
-    return cudaEventRecord(static_cast<cudaEvent_t>(stage_events[idx]), s) == cudaSuccess;
-  };
-  const mpm::AffinityTile tile = tile_of(algo);
-  cudaError_t e = cudaSuccess;
-  if (!mark(0)) return MPM_ERR_CUDA;
-  e = mpm::launch_prep(tokens, offsets, batch, rows, dim, bf16, tile, ws, sms, s);
-  if (e != cudaSuccess || !mark(1) || !mark(2)) return MPM_ERR_CUDA;
-  if (rows > 0) {
-    e = launch_affinity(algo, tokens, batch, rows, dim, bf16, ws, sms, s);
-    if (e != cudaSuccess) return MPM_ERR_CUDA;
-  }
-  if (!mark(3) || !mark(4)) return MPM_ERR_CUDA;
-  e = mpm::launch_mutual_compact(batch, ws, out_map, out_offsets, s);
-  if (e != cudaSuccess || !mark(5) || !mark(6)) return MPM_ERR_CUDA;
-  if (rows > 0) {
-    e = mpm::launch_pair_average(tokens, out_tokens, batch, rows, dim, bf16, ws, out_offsets, sms, s);
-    if (e != cudaSuccess) return MPM_ERR_CUDA;
-  }
-  return mark(7) ? MPM_OK : MPM_ERR_CUDA;
+  return merge_impl(tokens, offsets, batch, rows, dim, dtype, 0, out_tokens, out_offsets, out_map, workspace,
+                    workspace_bytes, stream, stage_events);
 }
 
 mpm_status mpm_merge(const void* tokens, const int64_t* offsets, int32_t batch, int64_t rows, int32_t dim,
                      mpm_dtype dtype, void* out_tokens, int64_t* out_offsets, int32_t* out_map, void* workspace,
                      size_t workspace_bytes, void* stream) {
-  return mpm_merge_timed(tokens, offsets, batch, rows, dim, dtype, out_tokens, out_offsets, out_map, workspace,
-                         workspace_bytes, stream, nullptr);
+  return merge_impl(tokens, offsets, batch, rows, dim, dtype, 0, out_tokens, out_offsets, out_map, workspace,
+                    workspace_bytes, stream, nullptr);
+}
+
+mpm_status mpm_merge_chunked(const void* tokens, const int64_t* offsets, int32_t batch, int64_t rows, int32_t dim,
+                             mpm_dtype dtype, int64_t chunk, void* out_tokens, int64_t* out_offsets,
+                             int32_t* out_map, void* workspace, size_t workspace_bytes, void* stream) {
+  return merge_impl(tokens, offsets, batch, rows, dim, dtype, chunk, out_tokens, out_offsets, out_map, workspace,
+                    workspace_bytes, stream, nullptr);
 }
 
 mpm_status mpm_compose_maps(const int32_t* map1, const int64_t* offsets0, int64_t rows0, const int32_t* map2,

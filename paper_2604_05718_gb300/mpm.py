@@ -28,7 +28,8 @@ STATUS_NAMES = {
 }
 EXPORTS = ("mpm_abi_version", "mpm_status_string", "mpm_merge_workspace_size", "mpm_merge", "mpm_merge_timed",
            "mpm_compose_maps", "mpm_unmerge_gather", "mpm_nearest_neighbors", "mpm_get_device_status",
-           "mpm_merge_no_alloc", "mpm_compose_gather", "mpm_pad_batch", "mpm_unpad_batch")
+           "mpm_merge_no_alloc", "mpm_compose_gather", "mpm_pad_batch", "mpm_unpad_batch", "mpm_merge_chunked",
+           "mpm_nearest_neighbors_chunked")
 
 _lib = None
 
@@ -58,6 +59,9 @@ def _declare(lib: ctypes.CDLL) -> None:
         "mpm_compose_gather": (ctypes.c_int, [P, P, I64, P, P, I64, P, P, I64, I32, I32, ctypes.c_int, P, P, P,
                                               P]),
         "mpm_pad_batch": (ctypes.c_int, [P, P, I32, I64, I32, ctypes.c_int, I64, P, P, P, P, P]),
+        "mpm_merge_chunked": (ctypes.c_int, [P, P, I32, I64, I32, ctypes.c_int, I64, P, P, P, P, SZ, P]),
+        "mpm_nearest_neighbors_chunked": (ctypes.c_int, [P, P, I32, I64, I32, ctypes.c_int, ctypes.c_int, I64, P, P,
+                                                         P, SZ, P]),
         "mpm_unpad_batch": (ctypes.c_int, [P, I32, I64, I32, ctypes.c_int, P, I64, P, P, P]),
     }
     for name, (res, args) in sigs.items():
@@ -132,7 +136,7 @@ def new_workspace(rows: int, batch: int, dim: int, dtype: torch.dtype, device) -
 
 def merge(tokens: torch.Tensor, offsets: torch.Tensor, workspace: torch.Tensor | None = None,
           out_tokens: torch.Tensor | None = None, out_offsets: torch.Tensor | None = None,
-          out_map: torch.Tensor | None = None, stage_events: list | None = None):
+          out_map: torch.Tensor | None = None, stage_events: list | None = None, chunk: int = 0):
     """One MPM call on a packed batch (Algorithm 1).
 
     tokens [rows, D] bf16/fp32 and offsets int64 [B+1] on the same GPU.
@@ -140,6 +144,8 @@ def merge(tokens: torch.Tensor, offsets: torch.Tensor, workspace: torch.Tensor |
     the first out_offsets[B] rows of out_tokens are the merged tokens.
     stage_events: optional 8 torch.cuda.Event (timing enabled, already
     recorded once so that they exist) bracketing the four kernels.
+    chunk: > 0 restricts every token's nearest-neighbour search to its run of
+    `chunk` consecutive tokens (mpm_merge_chunked; a multiple of 256).
     """
     _cuda(tokens, "tokens", ndim=2)
     _cuda(offsets, "offsets", torch.int64, 1)
@@ -159,17 +165,24 @@ def merge(tokens: torch.Tensor, offsets: torch.Tensor, workspace: torch.Tensor |
         if len(stage_events) != 8:
             raise ValueError("stage_events needs 8 events")
         events = (ctypes.c_void_p * 8)(*[ctypes.c_void_p(e.cuda_event) for e in stage_events])
+    if chunk and stage_events is not None:
+        raise ValueError("stage_events are only recorded by the unchunked merge")
     with torch.cuda.device(dev):
-        code = library().mpm_merge_timed(_ptr(tokens), _ptr(offsets), batch, rows, dim, _dtype_code(tokens),
-                                         _ptr(out_tokens), _ptr(out_offsets), _ptr(out_map), _ptr(workspace),
-                                         workspace.numel(), _stream(dev), events)
+        if chunk:
+            code = library().mpm_merge_chunked(_ptr(tokens), _ptr(offsets), batch, rows, dim, _dtype_code(tokens),
+                                               int(chunk), _ptr(out_tokens), _ptr(out_offsets), _ptr(out_map),
+                                               _ptr(workspace), workspace.numel(), _stream(dev))
+        else:
+            code = library().mpm_merge_timed(_ptr(tokens), _ptr(offsets), batch, rows, dim, _dtype_code(tokens),
+                                             _ptr(out_tokens), _ptr(out_offsets), _ptr(out_map), _ptr(workspace),
+                                             workspace.numel(), _stream(dev), events)
     _check("mpm_merge", code)
     return out_tokens, out_offsets, out_map
 
 
 def nearest_neighbors(tokens: torch.Tensor, offsets: torch.Tensor, algo: str = "auto",
-                      workspace: torch.Tensor | None = None, with_score: bool = True):
-    """b(i) (local index, -1 when alone) and its fp32 cosine, per token."""
+                      workspace: torch.Tensor | None = None, with_score: bool = True, chunk: int = 0):
+    """b(i) (local index, -1 when alone) and its fp32 cosine, per token (within chunks if chunk > 0)."""
     _cuda(tokens, "tokens", ndim=2)
     _cuda(offsets, "offsets", torch.int64, 1)
     dev = tokens.device
@@ -180,9 +193,15 @@ def nearest_neighbors(tokens: torch.Tensor, offsets: torch.Tensor, algo: str = "
     nn = torch.empty(rows, dtype=torch.int32, device=dev)
     score = torch.empty(rows, dtype=torch.float32, device=dev) if with_score else None
     with torch.cuda.device(dev):
-        code = library().mpm_nearest_neighbors(_ptr(tokens), _ptr(offsets), batch, rows, dim,
-                                               _dtype_code(tokens), ALGOS[algo], _ptr(nn), _ptr(score),
-                                               _ptr(workspace), workspace.numel(), _stream(dev))
+        if chunk:
+            code = library().mpm_nearest_neighbors_chunked(_ptr(tokens), _ptr(offsets), batch, rows, dim,
+                                                           _dtype_code(tokens), ALGOS[algo], int(chunk), _ptr(nn),
+                                                           _ptr(score), _ptr(workspace), workspace.numel(),
+                                                           _stream(dev))
+        else:
+            code = library().mpm_nearest_neighbors(_ptr(tokens), _ptr(offsets), batch, rows, dim,
+                                                   _dtype_code(tokens), ALGOS[algo], _ptr(nn), _ptr(score),
+                                                   _ptr(workspace), workspace.numel(), _stream(dev))
     _check("mpm_nearest_neighbors", code)
     return nn, score
 

@@ -95,14 +95,14 @@ def check_partition(nn: np.ndarray, rmap: np.ndarray, n: int, what: str) -> list
 
 
 def check_image(x: np.ndarray, nn_g: np.ndarray, map_g: np.ndarray, out_g: np.ndarray, dtype: str,
-                what: str) -> tuple:
+                what: str, chunk: int | None = None) -> tuple:
     """One image of one MPM call.  x: the exact stored input (fp64 values).
 
     Returns (stats, oracle MergeResult, exact) where exact is True when the
     GPU reproduced the oracle's nearest neighbours, map and features exactly.
     """
     st = ParityStats(images=1, rows=x.shape[0])
-    res = oracle.merge_image(x)
+    res = oracle.merge_image(x, chunk)
     n = x.shape[0]
     if n == 0:
         assert out_g.shape[0] == 0
@@ -116,7 +116,7 @@ def check_image(x: np.ndarray, nn_g: np.ndarray, map_g: np.ndarray, out_g: np.nd
         f"{np.nonzero(decisive_bad)[0][:5].tolist()}")
     differ = nn_g != res.nn.b
     if differ.any():
-        s = oracle.cosine_affinity(x)
+        s = oracle.cosine_affinity(x, chunk)
         for i in np.nonzero(differ)[0]:
             j = int(nn_g[i])
             assert 0 <= j < n and j != i, f"{what}: invalid neighbour {j} for row {i}"
@@ -141,7 +141,7 @@ def check_image(x: np.ndarray, nn_g: np.ndarray, map_g: np.ndarray, out_g: np.nd
 
 def check_merge_batch(x: np.ndarray, offsets: np.ndarray, gpu_nn: np.ndarray, gpu_map: np.ndarray,
                       gpu_out: np.ndarray, gpu_out_offsets: np.ndarray, dtype: str, what: str,
-                      images=None) -> ParityStats:
+                      images=None, chunk: int | None = None) -> ParityStats:
     """check_image over the (sampled) images of a packed batch."""
     st = ParityStats()
     assert gpu_out_offsets[0] == 0 and np.all(np.diff(gpu_out_offsets) >= 0)
@@ -149,6 +149,7 @@ def check_merge_batch(x: np.ndarray, offsets: np.ndarray, gpu_nn: np.ndarray, gp
     for b in idx:
         a0, a1 = offsets[b], offsets[b + 1]
         o0, o1 = gpu_out_offsets[b], gpu_out_offsets[b + 1]
-        s, _, _ = check_image(x[a0:a1], gpu_nn[a0:a1], gpu_map[a0:a1], gpu_out[o0:o1], dtype, f"{what}[{b}]")
+        s, _, _ = check_image(x[a0:a1], gpu_nn[a0:a1], gpu_map[a0:a1], gpu_out[o0:o1], dtype, f"{what}[{b}]",
+                              chunk)
         st.add(s)
     return st

@@ -137,4 +137,14 @@ def test_nn_compose_gather_validation(lib):
     assert unpad(P(FAKE), 2, 8, 64, 1, P(FAKE), 10, None, None, None) == 1                       # no output
     assert unpad(P(FAKE), 2, 8, 64, 1, P(FAKE), 10, P(FAKE + 128), None, None) == 8              # out overlaps padded
     assert unpad(P(FAKE), 2, 8, 60, 1, P(FAKE), 10, P(FAKE * 8), None, None) == 3                # 120-byte rows
+    mc = lib.mpm_merge_chunked
+    # (tokens, offsets, batch, rows, dim, dtype, chunk, out_tokens, out_offsets, out_map, workspace, bytes, stream)
+    args = (P(FAKE), P(FAKE), 1, 10, 64, 1)
+    outs = (P(FAKE * 8), P(FAKE * 16), P(FAKE * 24), P(FAKE * 32), 1 << 24, None)
+    assert mc(*args, -1, *outs) == 1     # negative chunk
+    assert mc(*args, 100, *outs) == 2    # not a whole number of 256-token tiles
+    nnc = lib.mpm_nearest_neighbors_chunked
+    # (tokens, offsets, batch, rows, dim, dtype, algo, chunk, out_nn, out_score, workspace, bytes, stream)
+    assert nnc(P(FAKE), P(FAKE), 1, 10, 64, 1, 2, 256, P(FAKE * 8), None, P(FAKE * 32), 1 << 24, None) == 2
+    assert nnc(P(FAKE), P(FAKE), 1, 10, 64, 1, 4, -256, P(FAKE * 8), None, P(FAKE * 32), 1 << 24, None) == 1
     assert lib.mpm_get_device_status(None, None, None) == 1

@@ -251,6 +251,67 @@ def test_batch_compose_gather_roundtrip():
         np.testing.assert_array_equal(up[a0:a1], z[m2.r[m1.out_offsets[b]:m1.out_offsets[b + 1]][m1.r[a0:a1]]])
 
 
+def test_chunked_hand():
+    # Four tokens in two chunks of 2: 0 and 2 are the same direction, but only
+    # pairs inside a chunk may form, so the pairs are (0, 1) and (2, 3).
+    x = np.array([[1.0, 0.0], [0.6, 0.8], [1.0, 0.01], [0.0, 1.0]])
+    full = mpm_oracle.merge_image(x)
+    assert full.nn.b.tolist() == [2, 3, 0, 1]
+    res = mpm_oracle.merge_image(x, chunk=2)
+    assert res.nn.b.tolist() == [1, 0, 3, 2]
+    assert res.r.tolist() == [0, 0, 1, 1]
+    # A token alone in its (last, shorter) chunk has no neighbour.
+    res3 = mpm_oracle.merge_image(x[:3], chunk=2)
+    assert res3.nn.b.tolist() == [1, 0, -1] and res3.r.tolist() == [0, 0, 1]
+
+
+@pytest.mark.parametrize("chunk", [3, 4, 7, 64])
+def test_chunked_is_per_chunk_merge(chunk):
+    """Pairs never cross chunks, so the chunked merge of an image is the merge of
+    each chunk on its own, the IDs of later chunks shifted by the earlier chunks' outputs."""
+    batch = make_custom([29], 12, "f32", seed=31)
+    x = batch.tokens.double().numpy()
+    got = mpm_oracle.merge_image(x, chunk=chunk)
+    xs, rs, shift = [], [], 0
+    for c0 in range(0, x.shape[0], chunk):
+        part = mpm_oracle.merge_image(x[c0:c0 + chunk])
+        xs.append(part.x_out)
+        rs.append(part.r + shift)
+        shift += part.n_out
+    np.testing.assert_array_equal(got.r, np.concatenate(rs))
+    np.testing.assert_array_equal(got.x_out, np.concatenate(xs))
+
+
+def test_chunked_exact_bruteforce_tiny():
+    """Exact rationals, chunk by chunk: every pick is an exact maximiser within its chunk."""
+    rng = np.random.default_rng(17)
+    checked = 0
+    for _ in range(200):
+        n = int(rng.integers(2, 10))
+        chunk = int(rng.integers(1, 6))
+        x = rng.integers(-3, 4, size=(n, 3))
+        got = mpm_oracle.merge_image(x.astype(np.float64), chunk=chunk)
+        for c0 in range(0, n, chunk):
+            part = x[c0:c0 + chunk].tolist()
+            if len(part) < 2:
+                assert got.nn.b[c0] == -1
+                continue
+            for i in range(len(part)):
+                j = int(got.nn.b[c0 + i])
+                assert c0 <= j < c0 + len(part), (part, i, j)
+                assert j - c0 in exact_maximisers(part, i), (part, i, j)
+                checked += 1
+    assert checked > 500
+
+
+def test_chunk_covering_the_image_is_the_full_merge():
+    batch = make_custom([40], 16, "f32", seed=32)
+    x = batch.tokens.double().numpy()
+    a, b = mpm_oracle.merge_image(x), mpm_oracle.merge_image(x, chunk=64)
+    np.testing.assert_array_equal(a.r, b.r)
+    np.testing.assert_array_equal(a.x_out, b.x_out)
+
+
 def test_pad_batch_hand():
     # Three images of 2, 0 and 3 one-feature tokens, padded to L = 3 (values written out by hand).
     x = np.array([[1.0], [2.0], [3.0], [4.0], [5.0]])
@@ -334,7 +395,7 @@ def _all_pins_pass() -> bool:
     return True
 
 
-def _nn_highest_tie(x, affinity=None):
+def _nn_highest_tie(x, affinity=None, chunk=None):
     nn = _orig_nn(x, affinity)
     n = np.asarray(x).shape[0]
     if n > 1:
@@ -343,13 +404,13 @@ def _nn_highest_tie(x, affinity=None):
     return nn
 
 
-def _nn_no_mask(x, affinity=None):
+def _nn_no_mask(x, affinity=None, chunk=None):
     xt = mpm_oracle.normalise_rows(x)
     s = xt @ xt.T
     return _orig_nn(x, s)
 
 
-def _nn_argmin(x, affinity=None):
+def _nn_argmin(x, affinity=None, chunk=None):
     n = np.asarray(x).shape[0]
     if n <= 1:
         return _orig_nn(x, affinity)
@@ -358,7 +419,7 @@ def _nn_argmin(x, affinity=None):
     return _orig_nn(x, -s)
 
 
-def _nn_unnormalised(x, affinity=None):
+def _nn_unnormalised(x, affinity=None, chunk=None):
     n = np.asarray(x).shape[0]
     if n <= 1:
         return _orig_nn(x, affinity)
