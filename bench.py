@@ -62,6 +62,7 @@ def parse_args():
     p.add_argument("--cpu-seconds", type=float, default=15.0, help="target CPU time of the oracle sample")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-chunked", action="store_true", help="skip the chunked-similarity measurement")
+    p.add_argument("--no-padded", action="store_true", help="skip the padded-batch measurement")
     return p.parse_args()
 
 
@@ -524,13 +525,14 @@ def run_mpm(args):
     # ---------------- padded batch of the stage-1 output (next-step consumer layout) ----------------
     # The merged sequences padded to the longest one, with a key mask, as the
     # paper batches them for dense attention; and back to the packed layout.
+    padded = None
     n1_max = int(n1.max())
-    pad_out = torch.empty(nimg, n1_max, dim, dtype=x1.dtype, device=dev)
+    pad_out = torch.empty(nimg, n1_max, dim, dtype=x1.dtype, device=dev) if not args.no_padded else None
     pad_mask = torch.empty(nimg, n1_max, dtype=torch.uint8, device=dev)
     pad_stats = torch.empty(3, dtype=torch.int64, device=dev)
-    unpadded = torch.empty_like(x1)
+    unpadded = torch.empty_like(x1) if not args.no_padded else None
     pad_us, unpad_us = [], []
-    for it in range(max(3, args.warmup) + 20):
+    for it in range(0 if args.no_padded else max(3, args.warmup) + 20):
         flush.fill_(1)
         flush_sum.copy_(flush.view(torch.int64).sum())
         e = new_events(3)
@@ -543,18 +545,19 @@ def run_mpm(args):
             torch.cuda.synchronize(dev)
             pad_us.append(1e3 * e[0].elapsed_time(e[1]))
             unpad_us.append(1e3 * e[1].elapsed_time(e[2]))
-    assert torch.equal(unpadded[:t1], x1[:t1]), "unpad(pad(x)) differs from x"
     hbm_bw = peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
     pad_bytes = float(n1.sum() * dim * esize + nimg * n1_max * (dim * esize + 1))
     unpad_bytes = float(2 * n1.sum() * dim * esize)
-    padded = {
-        "L": n1_max, "rows": int(n1.sum()), "padding_frac": 1.0 - float(n1.sum()) / (nimg * n1_max),
-        "pad_us": statistics.median(pad_us), "unpad_us": statistics.median(unpad_us),
-        "pad_gbs": pad_bytes / (statistics.median(pad_us) * 1e-6) / 1e9,
-        "unpad_gbs": unpad_bytes / (statistics.median(unpad_us) * 1e-6) / 1e9,
-    }
-    padded["pad_frac"] = padded["pad_gbs"] / hbm_bw
-    padded["unpad_frac"] = padded["unpad_gbs"] / hbm_bw
+    if not args.no_padded:
+        assert torch.equal(unpadded[:t1], x1[:t1]), "unpad(pad(x)) differs from x"
+        padded = {
+            "L": n1_max, "rows": int(n1.sum()), "padding_frac": 1.0 - float(n1.sum()) / (nimg * n1_max),
+            "pad_us": statistics.median(pad_us), "unpad_us": statistics.median(unpad_us),
+            "pad_gbs": pad_bytes / (statistics.median(pad_us) * 1e-6) / 1e9,
+            "unpad_gbs": unpad_bytes / (statistics.median(unpad_us) * 1e-6) / 1e9,
+        }
+        padded["pad_frac"] = padded["pad_gbs"] / hbm_bw
+        padded["unpad_frac"] = padded["unpad_gbs"] / hbm_bw
 
     # ---------------- chunked similarity on the mixed-resolution workload ----------------
     # One merge of the mixed workload (1024-4096 tokens per image) with the
