@@ -63,6 +63,7 @@ def parse_args():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-chunked", action="store_true", help="skip the chunked-similarity measurement")
     p.add_argument("--no-padded", action="store_true", help="skip the padded-batch measurement")
+    p.add_argument("--no-fp32", action="store_true", help="skip the fp32 nearest-neighbour measurement")
     return p.parse_args()
 
 
@@ -315,7 +316,7 @@ def run_mpm(args):
 
     import paper_2604_05718_gb300 as mpm
     from paper_2604_05718_gb300 import build
-    from workloads import CONFIGS, apply_noise, make_batch, stage_noise
+    from workloads import CONFIGS, WorkloadConfig, apply_noise, make_batch, stage_noise
 
     rank, world, local = dist_env()
     if not torch.cuda.is_available():
@@ -593,6 +594,39 @@ def run_mpm(args):
             "merged_tokens_full": res[0][1], "merged_tokens_chunk_1024": res[1024][1],
         }
 
+    # ---------------- fp32 tokens: three tf32 products on the tensor cores vs CUDA-core FMA ----------------
+    # The nearest-neighbour step (Eq. 1 + arg max) of the same image shapes
+    # in fp32, through MPM_NN_TCGEN05_PAIR (the fp32 default) and MPM_NN_SIMT.
+    fp32 = None
+    if rank == 0 and not args.no_fp32:
+        f_cfg = WorkloadConfig("vit_b_fp32", cfg.batch, cfg.sides, cfg.dim, "f32", cfg.k_range, cfg.sigma_range,
+                               cfg.insertions, cfg.seed)
+        fb = make_batch(f_cfg)
+        fx = fb.tokens.to(dev)
+        foff = torch.from_numpy(fb.offsets).to(dev)
+        fws = mpm.new_workspace(fb.rows, f_cfg.batch, f_cfg.dim, fx.dtype, dev)
+        f_us, f_nn = {}, {}
+        for algo in ("tcgen05_pair", "simt"):
+            ts = []
+            for it in range(max(3, args.warmup) + 10):
+                flush.fill_(1)
+                flush_sum.copy_(flush.view(torch.int64).sum())
+                e = new_events(2)
+                e[0].record(stream)
+                nn_f, _ = mpm.nearest_neighbors(fx, foff, algo=algo, workspace=fws, with_score=False)
+                e[1].record(stream)
+                if it >= max(3, args.warmup):
+                    torch.cuda.synchronize(dev)
+                    ts.append(1e3 * e[0].elapsed_time(e[1]))
+            f_us[algo] = statistics.median(ts)
+            f_nn[algo] = nn_f
+        fp32 = {
+            "workload": f"{f_cfg.batch} x {int(fb.offsets[1])} tokens x {f_cfg.dim} fp32 (vit_b shapes)",
+            "nn_us_tensor_3xtf32": f_us["tcgen05_pair"], "nn_us_simt_fma": f_us["simt"],
+            "speedup": f_us["simt"] / f_us["tcgen05_pair"],
+            "same_neighbour_frac": float((f_nn["tcgen05_pair"] == f_nn["simt"]).float().mean()),
+        }
+
     # ---------------- end to end: host buffers, copies inside the timed region ----------------
     # A serving loop: every step copies its tokens and offsets in from pinned
     # host memory, runs the whole step (L2 flush, merge, stand-in noise,
@@ -678,6 +712,7 @@ def run_mpm(args):
             "hbm_kernels": hbm_kernels,
             "padded_batch": padded,
             "chunked_similarity": chunked,
+            "fp32_nearest_neighbours": fp32,
             "kernels_us": kern,
             "ms_per_step_with_kernel_events": ms_with_kernel_events,
             "cpu_baseline": cpu_base,

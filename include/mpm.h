@@ -73,13 +73,16 @@ typedef enum mpm_status {
 
 /* Which kernel computes the nearest neighbours (Eq. 1 + arg max). */
 typedef enum mpm_nn_algo {
-  MPM_NN_AUTO = 0,         /* MPM_NN_TCGEN05_PAIR for bf16, MPM_NN_SIMT for fp32 */
+  MPM_NN_AUTO = 0,         /* MPM_NN_TCGEN05_PAIR (both dtypes) */
   MPM_NN_SIMT = 1,         /* CUDA-core fp32 FMA tiles (any dtype) */
   MPM_NN_TCGEN05 = 2,      /* TMA + tcgen05 MMA into TMEM, every tile of X X^T (bf16) */
   MPM_NN_TCGEN05_SYM = 3,  /* as above, tiles on or above the diagonal only, each
                               feeding both its rows and its columns (bf16) */
   MPM_NN_TCGEN05_PAIR = 4  /* symmetric, 256 x 256 tiles on SM pairs with
-                              tcgen05.mma.cta_group::2 (bf16) */
+                              tcgen05.mma.cta_group::2: bf16 products for bf16
+                              tokens; for fp32 tokens three tf32 products per
+                              term (x = hi + lo with hi the tf32 rounding of x:
+                              hi.hi + hi.lo + lo.hi, accumulated in fp32) */
 } mpm_nn_algo;
 
 /* Version of this ABI (MPM_ABI_VERSION). */
@@ -93,7 +96,8 @@ MPM_API const char* mpm_status_string(mpm_status status);
  * for `rows` token rows and `batch` images.  Returns 0 for invalid sizes.
  * The workspace must be 256-byte aligned.  It holds per-row inverse norms,
  * packed arg-max keys, the representative list, per-image counts, sanitised
- * offsets, the work plan and the device status word.
+ * offsets, the work plan and the device status word; for fp32 tokens also
+ * the tf32 high and low parts of the tokens (2 * rows * dim floats).
  */
 MPM_API size_t mpm_merge_workspace_size(int64_t rows, int32_t batch, int32_t dim, mpm_dtype dtype);
 
@@ -292,8 +296,8 @@ MPM_API mpm_status mpm_unpad_batch(const void* padded, int32_t batch, int64_t ma
  * Nearest neighbours only (Eq. 1 and Algorithm 1 step 3), for testing and
  * diagnostics.  out_nn int32 [rows]: local index b(i) (-1 for a token alone
  * in its image); out_score float [rows] (may be NULL): the cosine S_{i,b(i)}
- * as computed in fp32.  `algo` selects the kernel (MPM_NN_TCGEN05 requires
- * bf16).  Same workspace as mpm_merge.
+ * as computed in fp32.  `algo` selects the kernel (MPM_NN_TCGEN05 and
+ * MPM_NN_TCGEN05_SYM require bf16).  Same workspace as mpm_merge.
  */
 MPM_API mpm_status mpm_nearest_neighbors(const void* tokens, const int64_t* offsets, int32_t batch,
                                  int64_t rows, int32_t dim, mpm_dtype dtype,

@@ -62,6 +62,13 @@ static_assert(EPI_COLS <= HALF && HALF % EPI_COLS == 0, "a warp's columns lie in
 constexpr int THREADS = (2 + EPI_WARPS) * 32;
 constexpr uint32_t TMEM_COLS = 2 * TILE;
 constexpr uint32_t IDESC = ptx::idesc_bf16_f32(2 * HALF, TILE);
+// fp32 tokens: three tf32 products per K slice (hi hi + hi lo + lo hi, the
+// "3xTF32" split), with a stage of 32 features holding four 16 KiB slices:
+// A high, A low, B high, B low (one 128-byte swizzle row of fp32 each).
+constexpr int TF_BOX_K = 32;
+constexpr int TF_BK = TF_BOX_K;
+constexpr uint32_t IDESC_TF32 = ptx::idesc_tf32_f32(2 * HALF, TILE);
+static_assert(4 * ATOM_BYTES == STAGE_BYTES && HALF * TF_BOX_K * 4 == ATOM_BYTES, "same stage size for both paths");
 constexpr uint64_t WAIT_LIMIT_NS = 2000000000ull;
 constexpr int kMaxItems = 160;
 constexpr int kMaxStagedImages = 511;  // plan and offsets staged in shared memory up to this batch
@@ -205,6 +212,49 @@ __device__ __forceinline__ void mma_stage_full(uint32_t d_tmem, uint64_t a_desc,
       : "memory");
 }
 
+// The twelve MMAs of one full fp32 stage (32 features = four K = 8 slices of
+// 32 bytes), three tf32 products per slice, then the release commit.  The
+// stage's slices lie at a_desc (A high), +1024 (A low), +2048 (B high) and
+// +3072 (B low) in descriptor units of 16 bytes.
+__device__ __forceinline__ void mma_stage_tf32x3(uint32_t d_tmem, uint64_t a_desc, uint32_t idesc,
+                                                 uint32_t accumulate, uint64_t* release) {
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t.reg .b64 ah, al, bh, bl;\n\t"
+      "setp.ne.b32 p, %3, 0;\n\t"
+      "setp.ne.b32 q, %5, 0;\n\t"
+      "add.s64 al, %1, 1024;\n\tadd.s64 bh, %1, 2048;\n\tadd.s64 bl, %1, 3072;\n\t"
+      "tcgen05.mma.cta_group::2.kind::tf32 [%0], %1, bh, %2, p;\n\t"
+      "tcgen05.mma.cta_group::2.kind::tf32 [%0], %1, bl, %2, q;\n\t"
+      "tcgen05.mma.cta_group::2.kind::tf32 [%0], al, bh, %2, q;\n\t"
+      "add.s64 ah, %1, 2;\n\tadd.s64 al, %1, 1026;\n\tadd.s64 bh, %1, 2050;\n\tadd.s64 bl, %1, 3074;\n\t"
+      "tcgen05.mma.cta_group::2.kind::tf32 [%0], ah, bh, %2, q;\n\t"
+      "tcgen05.mma.cta_group::2.kind::tf32 [%0], ah, bl, %2, q;\n\t"
+      "tcgen05.mma.cta_group::2.kind::tf32 [%0], al, bh, %2, q;\n\t"
+      "add.s64 ah, %1, 4;\n\tadd.s64 al, %1, 1028;\n\tadd.s64 bh, %1, 2052;\n\tadd.s64 bl, %1, 3076;\n\t"
+      "tcgen05.mma.cta_group::2.kind::tf32 [%0], ah, bh, %2, q;\n\t"
+      "tcgen05.mma.cta_group::2.kind::tf32 [%0], ah, bl, %2, q;\n\t"
+      "tcgen05.mma.cta_group::2.kind::tf32 [%0], al, bh, %2, q;\n\t"
+      "add.s64 ah, %1, 6;\n\tadd.s64 al, %1, 1030;\n\tadd.s64 bh, %1, 2054;\n\tadd.s64 bl, %1, 3078;\n\t"
+      "tcgen05.mma.cta_group::2.kind::tf32 [%0], ah, bh, %2, q;\n\t"
+      "tcgen05.mma.cta_group::2.kind::tf32 [%0], ah, bl, %2, q;\n\t"
+      "tcgen05.mma.cta_group::2.kind::tf32 [%0], al, bh, %2, q;\n\t"
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%4], %6;\n\t}"
+      ::"r"(d_tmem), "l"(a_desc), "r"(idesc), "r"(accumulate), "r"(ptx::smem_addr(release)), "r"(1u),
+      "h"(static_cast<uint16_t>(3))
+      : "memory");
+}
+
+// One tf32 MMA (K = 8), issued by one thread.
+__device__ __forceinline__ void mma_pair_tf32(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                              uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::tf32 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
 // Arrives on the barrier at this offset in both CTAs once the MMAs issued so
 // far completed.
 __device__ __forceinline__ void commit_both(uint64_t* bar) {
@@ -224,8 +274,13 @@ __device__ __forceinline__ void fail(Control* ctl, int32_t* status, int32_t role
   report(status, MPM_ERR_DEVICE_TIMEOUT, role);
 }
 
+// TF32: fp32 tokens through the three-product tf32 split (tmap = high
+// parts, tmap_lo = low parts); otherwise bf16 tokens (tmap_lo unused).
+template <bool TF32>
 __global__ void __launch_bounds__(THREADS, 1)
-    affinity_pair_kernel(const __grid_constant__ CUtensorMap tmap, int batch, int dim, int64_t chunk, Workspace ws) {
+    affinity_pair_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constant__ CUtensorMap tmap_lo,
+                         int batch, int dim, int64_t chunk, Workspace ws) {
+  constexpr int kBK = TF32 ? TF_BK : BK;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024u - (ptx::smem_addr(smem_raw) & 1023u)) & 1023u);
   uint8_t* stages = smem;
@@ -239,7 +294,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = cluster_rank();
   const bool leader = rank == 0;
-  const int ksteps = (dim + BK - 1) / BK;
+  const int ksteps = (dim + kBK - 1) / kBK;
   const int64_t clusters = cluster_count();
   const int64_t cid = cluster_id();
 
@@ -316,10 +371,17 @@ __global__ void __launch_bounds__(THREADS, 1)
           uint8_t* sa = stages + stage * STAGE_BYTES;
           const uint32_t full_leader = map_to_rank(ptx::smem_addr(&ctl->full[stage]), 0);
           if (leader) ptx::mbar_arrive_expect_tx(&ctl->full[stage], 2 * STAGE_BYTES);
+          if constexpr (TF32) {
+            tma_load_2d_pair(sa, &tmap, full_leader, kb * kBK, arow);                    // A high
+            tma_load_2d_pair(sa + ATOM_BYTES, &tmap_lo, full_leader, kb * kBK, arow);    // A low
+            tma_load_2d_pair(sa + 2 * ATOM_BYTES, &tmap, full_leader, kb * kBK, brow);   // B high
+            tma_load_2d_pair(sa + 3 * ATOM_BYTES, &tmap_lo, full_leader, kb * kBK, brow);// B low
+          } else {
 #pragma unroll
-          for (int t = 0; t < ATOMS; ++t) {
-            tma_load_2d_pair(sa + t * ATOM_BYTES, &tmap, full_leader, kb * BK + t * BOX_K, arow);
-            tma_load_2d_pair(sa + SLICE_BYTES + t * ATOM_BYTES, &tmap, full_leader, kb * BK + t * BOX_K, brow);
+            for (int t = 0; t < ATOMS; ++t) {
+              tma_load_2d_pair(sa + t * ATOM_BYTES, &tmap, full_leader, kb * BK + t * BOX_K, arow);
+              tma_load_2d_pair(sa + SLICE_BYTES + t * ATOM_BYTES, &tmap, full_leader, kb * BK + t * BOX_K, brow);
+            }
           }
           issued |= 1 << stage;
           issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
@@ -359,7 +421,21 @@ __global__ void __launch_bounds__(THREADS, 1)
           }
           ptx::tc_fence_after_sync();
           const uint64_t a_desc = desc0 + static_cast<uint64_t>((stage * STAGE_BYTES) >> 4);
-          if ((kb + 1) * BK <= dim) {
+          if constexpr (TF32) {
+            if ((kb + 1) * kBK <= dim) {
+              mma_stage_tf32x3(d_tmem, a_desc, IDESC_TF32, kb != 0 ? 1u : 0u, &ctl->empty[stage]);
+            } else {
+              // Last, partial stage: the K = 8 slices that hold features.
+              for (int kk = 0; kk < kBK / 8 && kb * kBK + kk * 8 < dim; ++kk) {
+                const uint64_t ah = a_desc + 2 * kk, al = ah + (ATOM_BYTES >> 4);
+                const uint64_t bh = ah + 2 * (ATOM_BYTES >> 4), bl = ah + 3 * (ATOM_BYTES >> 4);
+                mma_pair_tf32(d_tmem, ah, bh, IDESC_TF32, (kb | kk) != 0 ? 1u : 0u);
+                mma_pair_tf32(d_tmem, ah, bl, IDESC_TF32, 1u);
+                mma_pair_tf32(d_tmem, al, bh, IDESC_TF32, 1u);
+              }
+              commit_both(&ctl->empty[stage]);
+            }
+          } else if ((kb + 1) * BK <= dim) {
             mma_stage_full(d_tmem, a_desc, IDESC, kb != 0 ? 1u : 0u, &ctl->empty[stage]);
           } else {
             // Last, partial stage: only the K slices that hold features.
@@ -493,29 +569,39 @@ PFN_cuTensorMapEncodeTiled_v12000 encoder() {
 
 AffinityTile pair_tile() { return {TILE, TILE, AffinityTile::kUpperSquare}; }
 
-cudaError_t launch_affinity_pair(const void* tokens, int batch, int64_t rows, int dim, int64_t chunk,
+cudaError_t launch_affinity_pair(const void* tokens, int batch, int64_t rows, int dim, bool tf32, int64_t chunk,
                                  const Workspace& ws, int num_sms, cudaStream_t stream) {
   PFN_cuTensorMapEncodeTiled_v12000 encode = encoder();
   if (encode == nullptr) return cudaErrorNotSupported;
-  CUtensorMap map;
+  // bf16: the tokens themselves; fp32: the tf32 high and low copies that the
+  // prep kernel wrote into the workspace.
+  const int esize = tf32 ? 4 : 2;
   const cuuint64_t gdim[2] = {static_cast<cuuint64_t>(dim), static_cast<cuuint64_t>(rows)};
-  const cuuint64_t gstride[1] = {static_cast<cuuint64_t>(dim) * 2};
-  const cuuint32_t box[2] = {BOX_K, HALF};
+  const cuuint64_t gstride[1] = {static_cast<cuuint64_t>(dim) * esize};
+  const cuuint32_t box[2] = {static_cast<cuuint32_t>(tf32 ? TF_BOX_K : BOX_K), HALF};
   const cuuint32_t estride[2] = {1, 1};
-  if (encode(&map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(tokens), gdim, gstride, box, estride,
-             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+  const CUtensorMapDataType type = tf32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+  void* hi = tf32 ? static_cast<void*>(ws.split_hi) : const_cast<void*>(tokens);
+  void* lo = tf32 ? static_cast<void*>(ws.split_lo) : const_cast<void*>(tokens);
+  if (hi == nullptr || lo == nullptr) return cudaErrorInvalidValue;
+  CUtensorMap map, map_lo;
+  if (encode(&map, type, 2, hi, gdim, gstride, box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
+             CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) !=
+          CUDA_SUCCESS ||
+      encode(&map_lo, type, 2, lo, gdim, gstride, box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
+             CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) !=
+          CUDA_SUCCESS)
     return cudaErrorInvalidValue;
-  static std::atomic<uint64_t> attr_done{0};
+  static std::atomic<uint64_t> attr_done[2] = {{0}, {0}};
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   const uint64_t bit = 1ull << (dev & 63);
-  if (!(attr_done.load() & bit)) {
-    e = cudaFuncSetAttribute(affinity_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(SMEM_BYTES));
+  auto kernel = tf32 ? affinity_pair_kernel<true> : affinity_pair_kernel<false>;
+  if (!(attr_done[tf32].load() & bit)) {
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(SMEM_BYTES));
     if (e != cudaSuccess) return e;
-    attr_done.fetch_or(bit);
+    attr_done[tf32].fetch_or(bit);
   }
   const int grid = (num_sms > 1 ? num_sms : 2) & ~1;  // whole SM pairs
   cudaLaunchConfig_t cfg = {};
@@ -532,7 +618,7 @@ cudaError_t launch_affinity_pair(const void* tokens, int batch, int64_t rows, in
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, affinity_pair_kernel, map, batch, dim, chunk, ws);
+  return cudaLaunchKernelEx(&cfg, kernel, map, map_lo, batch, dim, chunk, ws);
 }
 
 }  // namespace mpm

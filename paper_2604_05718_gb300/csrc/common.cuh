@@ -128,6 +128,30 @@ __device__ __forceinline__ float key_score(unsigned long long key) {
 // ---------------------------------------------------------------------------
 // 16-byte vectors: 8 bf16 or 4 fp32 lanes.
 // ---------------------------------------------------------------------------
+// x rounded to tf32 (10 explicit mantissa bits, round half to even); the
+// tensor core's kind::tf32 products use exactly these bits.  Values whose
+// rounding would overflow are truncated instead; infinities and NaNs pass.
+__device__ __forceinline__ float round_tf32(float x) {
+  const uint32_t u = __float_as_uint(x);
+  if ((u & 0x7F800000u) == 0x7F800000u) return x;
+  uint32_t r = (u + 0x0FFFu + ((u >> 13) & 1u)) & 0xFFFFE000u;
+  if ((r & 0x7F800000u) == 0x7F800000u) r = u & 0xFFFFE000u;
+  return __uint_as_float(r);
+}
+
+// Splits four fp32 values into tf32 high parts and the exact remainders
+// x - hi (hi + lo = x; lo is again rounded to tf32 by the products).
+__device__ __forceinline__ void split_tf32(uint4 v, uint4& hi, uint4& lo) {
+  const float* f = reinterpret_cast<const float*>(&v);
+  float* h = reinterpret_cast<float*>(&hi);
+  float* l = reinterpret_cast<float*>(&lo);
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    h[k] = round_tf32(f[k]);
+    l[k] = f[k] - h[k];
+  }
+}
+
 __device__ __forceinline__ float sumsq16(uint4 v, bool bf16) {
   float s = 0.f;
   if (bf16) {

@@ -36,6 +36,9 @@ struct ImageCursor {
 // Prep: status reset, offsets sanitisation + work plan (block 0), inverse
 // row norms and key reset (all blocks).
 // ---------------------------------------------------------------------------
+// SPLIT: also write the tf32 high / low parts of fp32 tokens (ws.split_hi /
+// split_lo) for the three-product tensor-core path.
+template <bool SPLIT>
 __global__ void __launch_bounds__(kThreads) prep_kernel(const uint8_t* __restrict__ tokens,
                                                         const int64_t* __restrict__ offsets,
                                                         int batch, int64_t rows, int row_bytes,
@@ -121,6 +124,21 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(const uint8_t* __restric
       for (int r = 0; r < kPrepRows; ++r)
 #pragma unroll
         for (int u = 0; u < kPrepVecs; ++u) s[r] += sumsq16(buf[r][u], bf16);
+      if constexpr (SPLIT) {
+#pragma unroll
+        for (int r = 0; r < kPrepRows; ++r)
+#pragma unroll
+          for (int u = 0; u < kPrepVecs; ++u) {
+            const int v = v0 + 32 * u;
+            if (g0 + r < used && v < nvec) {
+              uint4 hi, lo;
+              split_tf32(buf[r][u], hi, lo);
+              const int64_t at = (g0 + r) * (row_bytes >> 4) + v;
+              reinterpret_cast<uint4*>(ws.split_hi)[at] = hi;
+              reinterpret_cast<uint4*>(ws.split_lo)[at] = lo;
+            }
+          }
+      }
     }
 #pragma unroll
     for (int r = 0; r < kPrepRows; ++r) {
@@ -390,7 +408,10 @@ cudaError_t launch_prep(const void* tokens, const int64_t* offsets, int batch, i
                         bool bf16, AffinityTile tile, const Workspace& ws, int num_sms,
                         cudaStream_t stream) {
   const int row_bytes = dim * (bf16 ? 2 : 4);
-  return launch_dependent(prep_kernel, dim3(grid_for(num_sms, 8)), dim3(kThreads), 0, stream,
+  if (ws.split_hi != nullptr)
+    return launch_dependent(prep_kernel<true>, dim3(grid_for(num_sms, 8)), dim3(kThreads), 0, stream,
+                            static_cast<const uint8_t*>(tokens), offsets, batch, rows, row_bytes, bf16, tile, ws);
+  return launch_dependent(prep_kernel<false>, dim3(grid_for(num_sms, 8)), dim3(kThreads), 0, stream,
                           static_cast<const uint8_t*>(tokens), offsets, batch, rows, row_bytes, bf16, tile, ws);
 }
 

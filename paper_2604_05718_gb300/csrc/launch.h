@@ -20,6 +20,11 @@ struct Workspace {
   float* inv_norm;            // float[rows] 1 / max(|x_i|, 1e-12)
   unsigned long long* keys;   // u64[rows] packed (score, lowest j) arg-max keys
   int2* reps;                 // int2[rows] (representative, partner or -1), per image
+  // fp32 tokens only: x split into a tf32 high part and the fp32 remainder
+  // (float[rows * dim] each), for the three-product tf32 tensor-core path.
+  // Null for bf16.
+  float* split_hi;
+  float* split_lo;
 };
 
 // Tile of one affinity work item: rows x columns of the cosine matrix, and
@@ -55,7 +60,8 @@ AffinityTile tc_tile(bool symmetric);
 bool tc_available();
 
 // Symmetric affinity + arg max on SM pairs (tcgen05.mma.cta_group::2, bf16).
-cudaError_t launch_affinity_pair(const void* tokens, int batch, int64_t rows, int dim, int64_t chunk,
+// tf32: fp32 tokens through the three-product tf32 split (ws.split_hi / split_lo).
+cudaError_t launch_affinity_pair(const void* tokens, int batch, int64_t rows, int dim, bool tf32, int64_t chunk,
                                  const Workspace& ws, int num_sms, cudaStream_t stream);
 AffinityTile pair_tile();
 

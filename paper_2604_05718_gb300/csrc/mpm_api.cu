@@ -24,10 +24,11 @@ int elem_size(mpm_dtype dt) { return dt == MPM_BF16 ? 2 : 4; }
 bool valid_dtype(mpm_dtype dt) { return dt == MPM_F32 || dt == MPM_BF16; }
 
 struct Layout {
-  size_t status, soff, plan, count, inv_norm, keys, reps, total;
+  size_t status, soff, plan, count, inv_norm, keys, reps, split_hi, split_lo, total;
 };
 
-Layout layout(int64_t rows, int32_t batch) {
+// split_elems: rows * dim for fp32 tokens (the tf32 high / low copies), 0 for bf16.
+Layout layout(int64_t rows, int32_t batch, size_t split_elems) {
   Layout l{};
   size_t off = 0;
   l.status = off;
@@ -44,12 +45,20 @@ Layout layout(int64_t rows, int32_t batch) {
   off += round_up(sizeof(unsigned long long) * static_cast<size_t>(rows));
   l.reps = off;
   off += round_up(sizeof(int2) * static_cast<size_t>(rows));
+  l.split_hi = off;
+  off += round_up(sizeof(float) * split_elems);
+  l.split_lo = off;
+  off += round_up(sizeof(float) * split_elems);
   l.total = off;
   return l;
 }
 
-Workspace carve(void* base, int64_t rows, int32_t batch) {
-  const Layout l = layout(rows, batch);
+size_t split_elems(int64_t rows, int32_t dim, mpm_dtype dtype) {
+  return dtype == MPM_F32 ? static_cast<size_t>(rows) * static_cast<size_t>(dim) : 0;
+}
+
+Workspace carve(void* base, int64_t rows, int32_t batch, size_t split) {
+  const Layout l = layout(rows, batch, split);
   uint8_t* p = static_cast<uint8_t*>(base);
   Workspace ws;
   ws.status = reinterpret_cast<int32_t*>(p + l.status);
@@ -59,6 +68,8 @@ Workspace carve(void* base, int64_t rows, int32_t batch) {
   ws.inv_norm = reinterpret_cast<float*>(p + l.inv_norm);
   ws.keys = reinterpret_cast<unsigned long long*>(p + l.keys);
   ws.reps = reinterpret_cast<int2*>(p + l.reps);
+  ws.split_hi = split > 0 ? reinterpret_cast<float*>(p + l.split_hi) : nullptr;
+  ws.split_lo = split > 0 ? reinterpret_cast<float*>(p + l.split_lo) : nullptr;
   return ws;
 }
 
@@ -97,9 +108,16 @@ mpm_status check_tokens(const void* tokens, int64_t rows, int32_t dim, mpm_dtype
   return MPM_OK;
 }
 
-// Kernel used when the caller does not choose one: the symmetric tensor-core
-// kernel for bf16, CUDA-core fp32 FMA for fp32 (faithful to fp32 inputs).
-mpm_nn_algo default_algo(mpm_dtype dtype) { return dtype == MPM_BF16 ? MPM_NN_TCGEN05_PAIR : MPM_NN_SIMT; }
+// Kernel used when the caller does not choose one: the SM-pair tensor-core
+// kernel, with bf16 products for bf16 tokens and three tf32 products (high
+// and low parts, about fp32 accuracy) for fp32 tokens.
+mpm_nn_algo default_algo(mpm_dtype) { return MPM_NN_TCGEN05_PAIR; }
+
+// The workspace's tf32 split copies are filled only for the fp32 tensor-core path.
+Workspace for_algo(Workspace ws, mpm_nn_algo algo, mpm_dtype dtype) {
+  if (!(algo == MPM_NN_TCGEN05_PAIR && dtype == MPM_F32)) ws.split_hi = ws.split_lo = nullptr;
+  return ws;
+}
 
 bool is_tensor_core(mpm_nn_algo a) {
   return a == MPM_NN_TCGEN05 || a == MPM_NN_TCGEN05_SYM || a == MPM_NN_TCGEN05_PAIR;
@@ -125,7 +143,7 @@ mpm_status check_chunk(mpm_nn_algo algo, int64_t chunk) {
 
 cudaError_t launch_affinity(mpm_nn_algo a, const void* tokens, int batch, int64_t rows, int dim, bool bf16,
                             int64_t chunk, const Workspace& ws, int sms, cudaStream_t s) {
-  if (a == MPM_NN_TCGEN05_PAIR) return mpm::launch_affinity_pair(tokens, batch, rows, dim, chunk, ws, sms, s);
+  if (a == MPM_NN_TCGEN05_PAIR) return mpm::launch_affinity_pair(tokens, batch, rows, dim, !bf16, chunk, ws, sms, s);
   if (a == MPM_NN_TCGEN05 || a == MPM_NN_TCGEN05_SYM)
     return mpm::launch_affinity_tc(tokens, batch, rows, dim, a == MPM_NN_TCGEN05_SYM, ws, sms, s);
   return mpm::launch_affinity_simt(tokens, batch, dim, bf16, chunk, ws, sms, s);
@@ -134,13 +152,14 @@ cudaError_t launch_affinity(mpm_nn_algo a, const void* tokens, int batch, int64_
 // The affinity + arg max stage shared by the merge and nearest-neighbour
 // entry points.
 mpm_status run_affinity(const void* tokens, const int64_t* offsets, int32_t batch, int64_t rows, int32_t dim,
-                        mpm_dtype dtype, mpm_nn_algo algo, int64_t chunk, const Workspace& ws,
+                        mpm_dtype dtype, mpm_nn_algo algo, int64_t chunk, const Workspace& ws_all,
                         cudaStream_t stream) {
   const bool bf16 = dtype == MPM_BF16;
   if (algo == MPM_NN_AUTO) algo = default_algo(dtype);
   const bool tc = is_tensor_core(algo);
   if (algo != MPM_NN_SIMT && !tc) return MPM_ERR_INVALID_ARG;
-  if (tc && !bf16) return MPM_ERR_UNSUPPORTED;
+  if (tc && !bf16 && algo != MPM_NN_TCGEN05_PAIR) return MPM_ERR_UNSUPPORTED;
+  const Workspace ws = for_algo(ws_all, algo, dtype);
   const mpm_status cs = check_chunk(algo, chunk);
   if (cs != MPM_OK) return cs;
   if (tc && !mpm::tc_available()) return MPM_ERR_UNSUPPORTED;
@@ -159,10 +178,10 @@ mpm_status nearest_neighbors_impl(const void* tokens, const int64_t* offsets, in
   mpm_status st = check_tokens(tokens, rows, dim, dtype);
   if (st != MPM_OK) return st;
   if (workspace == nullptr || (reinterpret_cast<uintptr_t>(workspace) % kAlign) != 0 ||
-      workspace_bytes < layout(rows, batch).total)
+      workspace_bytes < layout(rows, batch, split_elems(rows, dim, dtype)).total)
     return MPM_ERR_WORKSPACE;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const Workspace ws = carve(workspace, rows, batch);
+  const Workspace ws = carve(workspace, rows, batch, split_elems(rows, dim, dtype));
   st = run_affinity(tokens, offsets, batch, rows, dim, dtype, algo, chunk, ws, s);
   if (st != MPM_OK) return st;
   return cuda_status(mpm::launch_decode_nn(batch, rows, ws, out_nn, out_score, num_sms(), s));
@@ -179,12 +198,12 @@ mpm_status merge_impl(const void* tokens, const int64_t* offsets, int32_t batch,
   const size_t bytes = static_cast<size_t>(rows) * dim * elem_size(dtype);
   if (overlap(tokens, bytes, out_tokens, bytes)) return MPM_ERR_ALIASING;
   if (workspace == nullptr || (reinterpret_cast<uintptr_t>(workspace) % kAlign) != 0 ||
-      workspace_bytes < layout(rows, batch).total)
+      workspace_bytes < layout(rows, batch, split_elems(rows, dim, dtype)).total)
     return MPM_ERR_WORKSPACE;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const Workspace ws = carve(workspace, rows, batch);
   const bool bf16 = dtype == MPM_BF16;
   const mpm_nn_algo algo = default_algo(dtype);
+  const Workspace ws = for_algo(carve(workspace, rows, batch, split_elems(rows, dim, dtype)), algo, dtype);
   st = check_chunk(algo, chunk);
   if (st != MPM_OK) return st;
   if (is_tensor_core(algo) && !mpm::tc_available()) return MPM_ERR_UNSUPPORTED;
@@ -237,7 +256,7 @@ const char* mpm_status_string(mpm_status status) {
 
 size_t mpm_merge_workspace_size(int64_t rows, int32_t batch, int32_t dim, mpm_dtype dtype) {
   if (!sizes_ok(rows, batch) || dim < 1 || !valid_dtype(dtype)) return 0;
-  return layout(rows, batch).total;
+  return layout(rows, batch, split_elems(rows, dim, dtype)).total;
 }
 
 mpm_status mpm_nearest_neighbors(const void* tokens, const int64_t* offsets, int32_t batch, int64_t rows,

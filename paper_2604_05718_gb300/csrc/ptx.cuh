@@ -136,6 +136,17 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(uint32_t m, uint32_t n) {
          | ((m >> 4) << 24);  // M >> 4
 }
 
+// Instruction descriptor of kind::tf32: tf32 A and B (fp32 bit patterns of
+// which the tensor core uses the top 19 bits), fp32 accumulator, K-major,
+// shape M x N.  Same fields as above with format code 2 (TF32) for A and B.
+__host__ __device__ constexpr uint32_t idesc_tf32_f32(uint32_t m, uint32_t n) {
+  return (1u << 4)            // D format: f32
+         | (2u << 7)          // A format: tf32
+         | (2u << 10)         // B format: tf32
+         | ((n >> 3) << 17)   // N >> 3
+         | ((m >> 4) << 24);  // M >> 4
+}
+
 // D[tmem] (+)= A[smem] * B[smem]^T for one K=16 slice, issued by one thread.
 __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
                                          uint32_t accumulate) {
