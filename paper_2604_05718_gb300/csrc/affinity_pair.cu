@@ -1,28 +1,31 @@
-// Symmetric affinity + arg max on SM pairs (bf16): the default kernel for
-// Eq. 1 and Algorithm 1 step 3.
+// Symmetric affinity + arg max on SM pairs: the default kernel for Eq. 1 and
+// Algorithm 1 step 3, for bf16 and fp32 tokens.
 //
-// Same arithmetic as affinity_tc.cu (raw bf16 dot products accumulated in
-// fp32 in tensor memory, scaled in fp32 by 1/max(|x|, 1e-12) in the
-// epilogue, packed (score, lowest index) keys merged with atomicMax), with
-// two changes in how the work is laid out:
+// Same arithmetic as affinity_tc.cu (raw dot products accumulated in fp32 in
+// tensor memory, scaled in fp32 by 1/max(|x|, 1e-12) in the epilogue, packed
+// (score, lowest index) keys merged with atomicMax), laid out as follows:
 //
 //  * A cluster of two CTAs (an SM pair) computes a 256 x 256 tile of
 //    G = X X^T with tcgen05.mma.cta_group::2 (M = 256, N = 256).  CTA r holds
 //    tile rows [128r, 128r + 128) of A and tile columns [128r, 128r + 128) of
 //    B in its own shared memory, and receives its 128 rows x 256 columns of
 //    the accumulator in its own tensor memory.  Each SM therefore stages 64
-//    KiB per 128-feature stage (two 64-feature TMA boxes per operand) instead
-//    of 96 KiB, which leaves room for three stages and cuts the
-//    shared-memory traffic of the tensor cores by a third.  The MMA warp
-//    issues a whole stage (eight MMAs and the release commit) from one asm
-//    block: its sub-partition also runs four epilogue warps, and every
+//    KiB per stage instead of 96 KiB, which leaves room for three stages and
+//    cuts the shared-memory traffic of the tensor cores by a third.
+//  * bf16 tokens: a stage holds 128 features (two 64-feature TMA boxes per
+//    operand) and takes eight K = 16 MMAs.  fp32 tokens (TF32 = true): every
+//    value is split as x = hi + lo (hi the tf32 rounding of x, written with
+//    lo by the prep kernel), a stage holds 32 features of A hi, A lo, B hi
+//    and B lo, and takes twelve K = 8 tf32 MMAs: hi.hi + hi.lo + lo.hi.
+//    The MMA warp issues a whole stage and its release commit from one asm
+//    block: its sub-partition also runs two epilogue warps, and every
 //    instruction it saves per stage keeps the tensor core fed.
 //  * Tiles are the 256 x 256 blocks on or above the diagonal of each image's
-//    G, R(R + 1) / 2 of them for R = ceil(N_b / 256).  Within a tile, every
-//    128-column block above a thread's 128-row block also yields column
-//    candidates (row j scores row i by G_ij / |x_i|), as in affinity_tc.cu's
-//    symmetric mode; the block below the diagonal of a diagonal tile is
-//    skipped.
+//    G (of each chunk's, with the chunked similarity), R(R + 1) / 2 of them
+//    for R = ceil(N / 256).  Within a tile, every 128-column block above a
+//    thread's 128-row block also yields column candidates (row j scores row
+//    i by G_ij / |x_i|), as in affinity_tc.cu's symmetric mode; the block
+//    below the diagonal of a diagonal tile is skipped.
 //
 // Roles per CTA (10 warps): warp 0 loads its CTA's A and B slices with TMA
 // and reports the bytes to the leader CTA's barrier; in the leader, warp 1
