@@ -36,6 +36,20 @@ inline cudaError_t launch_dependent(void (*kernel)(Params...), dim3 grid, dim3 b
   return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
 }
 
+// Blocks of `threads` threads of `kernel` that one SM holds at once
+// (registers and static shared memory permitting), at most `cap`.  The
+// bandwidth-bound kernels stride over rows with num_sms times this many
+// blocks: one wave, so no block waits for another to retire before its
+// share of the rows starts streaming (measured: a 2-wave grid of the same
+// kernels made the vit_b step 2% slower).  Occupancy depends only on the
+// kernel and the architecture, so callers keep the answer in a static.
+template <typename... Params>
+inline int resident_per_sm(void (*kernel)(Params...), int threads, int cap) {
+  int n = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kernel, threads, 0) != cudaSuccess || n < 1) return cap;
+  return n < cap ? n : cap;
+}
+
 // First error wins; `st` may be null (not reported).
 __device__ __forceinline__ void report(int32_t* st, int32_t code, int32_t detail) {
   if (st != nullptr && atomicCAS(st, 0, code) == 0) st[1] = detail;

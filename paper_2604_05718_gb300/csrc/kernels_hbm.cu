@@ -408,10 +408,13 @@ cudaError_t launch_prep(const void* tokens, const int64_t* offsets, int batch, i
                         bool bf16, AffinityTile tile, const Workspace& ws, int num_sms,
                         cudaStream_t stream) {
   const int row_bytes = dim * (bf16 ? 2 : 4);
-  if (ws.split_hi != nullptr)
-    return launch_dependent(prep_kernel<true>, dim3(grid_for(num_sms, 8)), dim3(kThreads), 0, stream,
+  if (ws.split_hi != nullptr) {
+    static const int per_sm = resident_per_sm(prep_kernel<true>, kThreads, 8);
+    return launch_dependent(prep_kernel<true>, dim3(grid_for(num_sms, per_sm)), dim3(kThreads), 0, stream,
                             static_cast<const uint8_t*>(tokens), offsets, batch, rows, row_bytes, bf16, tile, ws);
-  return launch_dependent(prep_kernel<false>, dim3(grid_for(num_sms, 8)), dim3(kThreads), 0, stream,
+  }
+  static const int per_sm = resident_per_sm(prep_kernel<false>, kThreads, 8);
+  return launch_dependent(prep_kernel<false>, dim3(grid_for(num_sms, per_sm)), dim3(kThreads), 0, stream,
                           static_cast<const uint8_t*>(tokens), offsets, batch, rows, row_bytes, bf16, tile, ws);
 }
 
@@ -425,7 +428,8 @@ cudaError_t launch_pair_average(const void* tokens, void* out_tokens, int batch,
                                 int dim, bool bf16, const Workspace& ws,
                                 const int64_t* out_offsets, int num_sms, cudaStream_t stream) {
   const int row_bytes = dim * (bf16 ? 2 : 4);
-  return launch_dependent(pair_average_kernel<1, 4>, dim3(grid_for(num_sms, 8)), dim3(kThreads), 0, stream,
+  static const int per_sm = resident_per_sm(pair_average_kernel<1, 4>, kThreads, 8);
+  return launch_dependent(pair_average_kernel<1, 4>, dim3(grid_for(num_sms, per_sm)), dim3(kThreads), 0, stream,
                           static_cast<const uint8_t*>(tokens), static_cast<uint8_t*>(out_tokens), batch, rows,
                           row_bytes, bf16, ws, out_offsets);
 }
@@ -449,7 +453,8 @@ cudaError_t launch_gather(const void* merged, const int64_t* moff, int64_t merge
                           int dim, bool bf16, void* out, int32_t* status, int num_sms,
                           cudaStream_t stream) {
   const int row_bytes = dim * (bf16 ? 2 : 4);
-  return launch_dependent(gather_kernel<3, 4, false>, dim3(grid_for(num_sms, 8)), dim3(kThreads), 0, stream,
+  static const int per_sm = resident_per_sm(gather_kernel<3, 4, false>, kThreads, 8);
+  return launch_dependent(gather_kernel<3, 4, false>, dim3(grid_for(num_sms, per_sm)), dim3(kThreads), 0, stream,
                           static_cast<const uint8_t*>(merged), moff, merged_rows, map, goff, grid_rows,
                           static_cast<const int32_t*>(nullptr), static_cast<const int64_t*>(nullptr),
                           static_cast<int64_t>(0), static_cast<int32_t*>(nullptr), batch, row_bytes,
@@ -462,7 +467,8 @@ cudaError_t launch_compose_gather(const void* merged, const int64_t* moff, int64
                                   bool bf16, void* out, int32_t* out_map, int32_t* status, int num_sms,
                                   cudaStream_t stream) {
   const int row_bytes = dim * (bf16 ? 2 : 4);
-  return launch_dependent(gather_kernel<3, 4, true>, dim3(grid_for(num_sms, 8)), dim3(kThreads), 0, stream,
+  static const int per_sm = resident_per_sm(gather_kernel<3, 4, true>, kThreads, 8);
+  return launch_dependent(gather_kernel<3, 4, true>, dim3(grid_for(num_sms, per_sm)), dim3(kThreads), 0, stream,
                           static_cast<const uint8_t*>(merged), moff, merged_rows, map1, off0, rows0, map2, off1,
                           rows1, out_map, batch, row_bytes, static_cast<uint8_t*>(out), status);
 }

@@ -127,7 +127,7 @@ __global__ void __launch_bounds__(kThreads) unpad_kernel(const uint8_t* __restri
   }
 }
 
-int pad_grid(int num_sms) { return (num_sms > 0 ? num_sms : 1) * 8; }
+int pad_grid(int num_sms, int per_sm) { return (num_sms > 0 ? num_sms : 1) * per_sm; }
 
 }  // namespace
 
@@ -135,7 +135,8 @@ cudaError_t launch_pad(const void* tokens, const int64_t* offsets, int batch, in
                        int dim, bool bf16, void* out, uint8_t* mask, int64_t* stats, int32_t* status, int num_sms,
                        cudaStream_t stream) {
   const int row_bytes = dim * (bf16 ? 2 : 4);
-  return launch_dependent(pad_kernel, dim3(pad_grid(num_sms)), dim3(kThreads), 0, stream,
+  static const int per_sm = resident_per_sm(pad_kernel, kThreads, 8);
+  return launch_dependent(pad_kernel, dim3(pad_grid(num_sms, per_sm)), dim3(kThreads), 0, stream,
                           static_cast<const uint8_t*>(tokens), offsets, batch, rows, max_len, row_bytes,
                           static_cast<uint8_t*>(out), mask, stats, status);
 }
@@ -143,7 +144,8 @@ cudaError_t launch_pad(const void* tokens, const int64_t* offsets, int batch, in
 cudaError_t launch_unpad(const void* padded, int batch, int64_t max_len, const int64_t* offsets, int64_t rows,
                          int dim, bool bf16, void* out, int32_t* status, int num_sms, cudaStream_t stream) {
   const int row_bytes = dim * (bf16 ? 2 : 4);
-  return launch_dependent(unpad_kernel, dim3(pad_grid(num_sms)), dim3(kThreads), 0, stream,
+  static const int per_sm = resident_per_sm(unpad_kernel, kThreads, 8);
+  return launch_dependent(unpad_kernel, dim3(pad_grid(num_sms, per_sm)), dim3(kThreads), 0, stream,
                           static_cast<const uint8_t*>(padded), batch, max_len, offsets, rows, row_bytes,
                           static_cast<uint8_t*>(out), status);
 }
