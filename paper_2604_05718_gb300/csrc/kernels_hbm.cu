@@ -13,7 +13,7 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kPrepRows = 2;   // rows per warp iteration in prep_kernel
-constexpr int kPrepVecs = 4;   // 16-byte vectors per lane and row per pass
+constexpr int kPrepVecs = 3;   // 16-byte vectors per lane and row per pass (one pass at D = 768 bf16)
 
 __device__ __forceinline__ int64_t clamp64(int64_t v, int64_t lo, int64_t hi) {
   return v < lo ? lo : (v > hi ? hi : v);
