@@ -140,6 +140,14 @@ def test_large_dim_and_large_image(mpm, algo):
     merge_parity(mpm, big, "n=6000", algo=algo)
 
 
+@pytest.mark.parametrize("algo", ["tcgen05_pair", "simt"])
+def test_rows_longer_than_a_prep_stage(mpm, algo):
+    # 24 KiB bf16 rows: prep reads them with plain loads instead of staging
+    # them through a 16 KiB shared-memory chunk.
+    batch = make_custom([70, 33], 12288, "bf16", seed=43)
+    merge_parity(mpm, batch, "d=12288", algo=algo)
+
+
 def test_tcgen05_and_simt_agree(mpm):
     batch = make_custom([1000, 513, 64, 2300], 384, "bf16", seed=9)
     runs = {algo: run_merge(mpm, batch.tokens, batch.offsets, algo)
