@@ -148,6 +148,17 @@ def test_rows_longer_than_a_prep_stage(mpm, algo):
     merge_parity(mpm, batch, "d=12288", algo=algo)
 
 
+@pytest.mark.parametrize("algo", ["tcgen05_pair", "simt"])
+def test_many_tiny_images(mpm, algo):
+    # 16,000 images of 0-5 tokens, one tile each: more images than the
+    # SM-pair kernel keeps in shared memory (511) and more tiles per pair of
+    # SMs than it decodes up front (160).
+    rng = np.random.default_rng(44)
+    counts = rng.choice([0, 1, 2, 3, 5], size=16000, p=[0.05, 0.2, 0.25, 0.25, 0.25]).tolist()
+    batch = make_custom(counts, 16, "bf16", seed=44)
+    merge_parity(mpm, batch, "16000 tiny images", algo=algo)
+
+
 def test_tcgen05_and_simt_agree(mpm):
     batch = make_custom([1000, 513, 64, 2300], 384, "bf16", seed=9)
     runs = {algo: run_merge(mpm, batch.tokens, batch.offsets, algo)
