@@ -321,6 +321,20 @@ MPM_API mpm_status mpm_nearest_neighbors_chunked(const void* tokens, const int64
  */
 MPM_API mpm_status mpm_get_device_status(void* workspace, int32_t* host_code, void* stream);
 
+/*
+ * Self-test of the device timeout path (the paper has no counterpart).
+ * Launches one block whose threads wait on an mbarrier that nothing ever
+ * completes, with the bounded wait (wall-time limit plus a probe cap) that
+ * the tensor-core kernels use on their pipeline barriers.  After limit_us
+ * microseconds the kernel records MPM_ERR_DEVICE_TIMEOUT in
+ * device_status[0] (detail 99 in device_status[1], first error wins, as in
+ * every MPM kernel) and returns; the CUDA context stays usable.
+ *   device_status  device int32[2], caller-owned, zeroed by the caller
+ *   limit_us       1 .. 10,000,000 (else MPM_ERR_INVALID_ARG)
+ * Asynchronous on `stream`.
+ */
+MPM_API mpm_status mpm_selftest_wait_timeout(int32_t* device_status, uint32_t limit_us, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

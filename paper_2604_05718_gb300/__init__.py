@@ -15,6 +15,7 @@ from .mpm import (  # noqa: F401
     nearest_neighbors,
     new_workspace,
     pad_batch,
+    selftest_wait_timeout,
     unmerge_gather,
     unpad_batch,
     workspace_size,

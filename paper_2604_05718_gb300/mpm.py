@@ -63,6 +63,7 @@ def _declare(lib: ctypes.CDLL) -> None:
         "mpm_nearest_neighbors_chunked": (ctypes.c_int, [P, P, I32, I64, I32, ctypes.c_int, ctypes.c_int, I64, P, P,
                                                          P, SZ, P]),
         "mpm_unpad_batch": (ctypes.c_int, [P, I32, I64, I32, ctypes.c_int, P, I64, P, P, P]),
+        "mpm_selftest_wait_timeout": (ctypes.c_int, [P, ctypes.c_uint32, P]),
     }
     for name, (res, args) in sigs.items():
         fn = getattr(lib, name)
@@ -349,3 +350,16 @@ def merge_no_alloc(tokens: torch.Tensor, offsets: torch.Tensor, out_tokens: torc
                                             _ptr(out_map), _stream(dev))
     _check("mpm_merge_no_alloc", code)
     return out_tokens, out_offsets, out_map
+
+
+def selftest_wait_timeout(limit_us: int, device=None) -> torch.Tensor:
+    """Runs the device timeout self-test (mpm_selftest_wait_timeout): a
+    bounded wait on a barrier that nothing completes.  Returns the int32[2]
+    device status word it wrote ([MPM_ERR_DEVICE_TIMEOUT, 99] when the wait
+    gave up as it should); the caller synchronises before reading it."""
+    dev = torch.device(device) if device is not None else torch.device("cuda", torch.cuda.current_device())
+    status = torch.zeros(2, dtype=torch.int32, device=dev)
+    with torch.cuda.device(dev):
+        code = library().mpm_selftest_wait_timeout(_ptr(status), int(limit_us), _stream(dev))
+    _check("mpm_selftest_wait_timeout", code)
+    return status
