@@ -4,6 +4,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include <atomic>
 
 #include "mpm.h"
@@ -12,6 +14,16 @@
 namespace {
 
 using mpm::Workspace;
+
+// Host-side NVTX range around one launch or one entry point (a profiler
+// can select an MPM stage by name; without a tool attached a range costs a
+// pointer check).
+struct Range {
+  explicit Range(const char* name) { nvtxRangePushA(name); }
+  ~Range() { nvtxRangePop(); }
+  Range(const Range&) = delete;
+  Range& operator=(const Range&) = delete;
+};
 
 constexpr size_t kAlign = 256;
 // Chunks of the chunked similarity are whole tiles of the SM-pair kernel.
@@ -216,17 +228,26 @@ mpm_status merge_impl(const void* tokens, const int64_t* offsets, int32_t batch,
   };
   const mpm::AffinityTile tile = tile_of(algo, chunk);
   cudaError_t e = cudaSuccess;
+  const Range whole("mpm_merge");
   if (!mark(0)) return MPM_ERR_CUDA;
-  e = mpm::launch_prep(tokens, offsets, batch, rows, dim, bf16, tile, ws, sms, s);
+  {
+    const Range r("mpm.prep");
+    e = mpm::launch_prep(tokens, offsets, batch, rows, dim, bf16, tile, ws, sms, s);
+  }
   if (e != cudaSuccess || !mark(1) || !mark(2)) return MPM_ERR_CUDA;
   if (rows > 0) {
+    const Range r("mpm.affinity");
     e = launch_affinity(algo, tokens, batch, rows, dim, bf16, chunk, ws, sms, s);
     if (e != cudaSuccess) return MPM_ERR_CUDA;
   }
   if (!mark(3) || !mark(4)) return MPM_ERR_CUDA;
-  e = mpm::launch_mutual_compact(batch, chunk, ws, out_map, out_offsets, s);
+  {
+    const Range r("mpm.mutual_scan");
+    e = mpm::launch_mutual_compact(batch, chunk, ws, out_map, out_offsets, s);
+  }
   if (e != cudaSuccess || !mark(5) || !mark(6)) return MPM_ERR_CUDA;
   if (rows > 0) {
+    const Range r("mpm.pair_average");
     e = mpm::launch_pair_average(tokens, out_tokens, batch, rows, dim, bf16, ws, out_offsets, sms, s);
     if (e != cudaSuccess) return MPM_ERR_CUDA;
   }
@@ -299,6 +320,7 @@ mpm_status mpm_merge_chunked(const void* tokens, const int64_t* offsets, int32_t
 mpm_status mpm_compose_maps(const int32_t* map1, const int64_t* offsets0, int64_t rows0, const int32_t* map2,
                             const int64_t* offsets1, int64_t rows1, int32_t batch, int32_t* out_map,
                             int32_t* device_status, void* stream) {
+  const Range whole("mpm_compose_maps");
   if (!sizes_ok(rows0, batch) || !sizes_ok(rows1, batch) || offsets0 == nullptr || offsets1 == nullptr)
     return MPM_ERR_INVALID_ARG;
   if (rows0 == 0) return MPM_OK;
@@ -313,6 +335,7 @@ mpm_status mpm_compose_maps(const int32_t* map1, const int64_t* offsets0, int64_
 mpm_status mpm_unmerge_gather(const void* merged, const int64_t* merged_offsets, int64_t merged_rows,
                               const int32_t* map, const int64_t* grid_offsets, int64_t grid_rows, int32_t batch,
                               int32_t dim, mpm_dtype dtype, void* out, int32_t* device_status, void* stream) {
+  const Range whole("mpm_unmerge_gather");
   if (!sizes_ok(merged_rows, batch) || !sizes_ok(grid_rows, batch) || merged_offsets == nullptr ||
       grid_offsets == nullptr)
     return MPM_ERR_INVALID_ARG;
@@ -334,6 +357,7 @@ mpm_status mpm_compose_gather(const void* merged, const int64_t* merged_offsets,
                               const int32_t* map1, const int64_t* offsets0, int64_t rows0, const int32_t* map2,
                               const int64_t* offsets1, int64_t rows1, int32_t batch, int32_t dim, mpm_dtype dtype,
                               void* out, int32_t* out_map, int32_t* device_status, void* stream) {
+  const Range whole("mpm_compose_gather");
   if (!sizes_ok(merged_rows, batch) || !sizes_ok(rows0, batch) || !sizes_ok(rows1, batch) ||
       merged_offsets == nullptr || offsets0 == nullptr || offsets1 == nullptr)
     return MPM_ERR_INVALID_ARG;
