@@ -148,6 +148,14 @@ def test_rows_longer_than_a_prep_stage(mpm, algo):
     merge_parity(mpm, batch, "d=12288", algo=algo)
 
 
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_maximum_dim(mpm, dtype):
+    # D = MPM_MAX_DIM = 16384: 32 KiB bf16 / 64 KiB fp32 rows, every K
+    # stage of the default kernels (the fp32 one through its tf32 split).
+    batch = make_custom([40, 17, 1], 16384, dtype, seed=45)
+    merge_parity(mpm, batch, f"d=16384 {dtype}")
+
+
 @pytest.mark.parametrize("algo", ["tcgen05_pair", "simt"])
 def test_many_tiny_images(mpm, algo):
     # 16,000 images of 0-5 tokens, one tile each: more images than the
