@@ -64,6 +64,9 @@ def parse_args():
     p.add_argument("--no-chunked", action="store_true", help="skip the chunked-similarity measurement")
     p.add_argument("--no-padded", action="store_true", help="skip the padded-batch measurement")
     p.add_argument("--no-fp32", action="store_true", help="skip the fp32 nearest-neighbour measurement")
+    p.add_argument("--timeline", action="store_true",
+                   help="instead of the benchmark, print each kernel's in-step duration from the device "
+                        "timeline of the traced library (libmpm_trace.so); one GPU")
     return p.parse_args()
 
 
@@ -729,10 +732,118 @@ def run_mpm(args):
     return 0
 
 
+# ---------------------------------------------------------------------------
+# Device timeline of the step (traced library)
+# ---------------------------------------------------------------------------
+def run_timeline(args):
+    """The benchmark step with the device timeline of libmpm_trace.so: for
+    every kernel, the time from the moment its blocks passed their wait for
+    the previous kernel to its last warp's end (GPU global timer), and the gap
+    since the previous kernel ended.  Inside the step, without the CUDA events
+    between kernels that the per-kernel figures of the benchmark need."""
+    import torch
+
+    import paper_2604_05718_gb300 as mpm
+    from paper_2604_05718_gb300 import build
+    from workloads import CONFIGS, apply_noise, make_batch, stage_noise
+
+    _, world, _ = dist_env()
+    if world > 1:
+        raise RuntimeError("--timeline runs on one GPU")
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    mpm.library(build.build(trace=True))
+    cfg = CONFIGS[args.workload]
+    batch = make_batch(cfg)
+    dim, esize = cfg.dim, (2 if cfg.dtype == "bf16" else 4)
+    two = cfg.insertions == 2
+    x0 = batch.tokens.to(dev)
+    off0 = torch.from_numpy(batch.offsets).to(dev)
+    ws = mpm.new_workspace(batch.rows, cfg.batch, dim, x0.dtype, dev)
+    x1, off1, m1 = mpm.merge(x0, off0, workspace=ws)
+    off1_h = off1.cpu().numpy()
+    t1 = int(off1_h[-1])
+    noise = stage_noise(cfg.seed, np.diff(off1_h).tolist(), dim).to(dev) if two else None
+    x1n = torch.zeros_like(x1)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    flush_sum = torch.zeros((), dtype=torch.int64, device=dev)
+    rows = {}
+    order = []
+
+    def record(stage, tl, prev_end):
+        for kind in ("prep", "affinity", "mutual_scan", "pair_average", "gather", "compose"):
+            if kind not in tl:
+                continue
+            start, waited, end = tl[kind]
+            key = f"{kind}_{stage}" if kind not in ("gather", "compose") else kind
+            if key not in rows:
+                rows[key] = []
+                order.append(key)
+            rows[key].append(((end - waited) * 1e-3, (end - start) * 1e-3,
+                              (waited - prev_end) * 1e-3 if prev_end else float("nan")))
+            prev_end = end
+        return prev_end
+
+    for it in range(args.warmup + args.steps):
+        flush.fill_(1)
+        flush_sum.copy_(flush.view(torch.int64).sum())
+        mpm.trace_reset()
+        x1, off1, m1 = mpm.merge(x0, off0, workspace=ws)
+        tl1 = mpm.trace_read()
+        if two:
+            x1n[:t1] = apply_noise(x1[:t1], noise)
+            torch.cuda.synchronize(dev)
+            mpm.trace_reset()
+            x2, off2, m2 = mpm.merge(x1n, off1, workspace=ws)
+            mpm.compose_gather(x2, off2, m1, off0, m2, off1)
+        else:
+            mpm.trace_reset()
+            mpm.unmerge_gather(x1, off1, m1, off0)
+        tl2 = mpm.trace_read()
+        if it >= args.warmup:
+            record(1, tl1, 0)
+            record(2, tl2, 0)
+    n0 = np.diff(batch.offsets).astype(np.float64)
+    n1 = np.diff(off1_h).astype(np.float64)
+    n2 = np.diff(off2.cpu().numpy()).astype(np.float64) if two else n1
+    hbm_bytes = {
+        "prep_1": n0.sum() * dim * esize + 12 * n0.sum(),
+        "prep_2": n1.sum() * dim * esize + 12 * n1.sum(),
+        "pair_average_1": (n0.sum() + n1.sum()) * dim * esize + 12 * n0.sum(),
+        "pair_average_2": (n1.sum() + n2.sum()) * dim * esize + 12 * n1.sum(),
+        "gather": (n2.sum() + n0.sum()) * dim * esize + (12 if two else 4) * n0.sum(),
+    }
+    flops = {"affinity_1": float(np.sum(n0 * (n0 - 1) * dim)), "affinity_2": float(np.sum(n1 * (n1 - 1) * dim))}
+    peaks, peak_kind = load_peaks()
+    out = {}
+    for key in order:
+        run = np.array(rows[key])
+        med = float(np.median(run[:, 0]))
+        entry = {"us_after_wait": med, "us_from_first_block": float(np.median(run[:, 1])),
+                 "gap_us_after_previous_kernel": float(np.nanmedian(run[:, 2])) if np.isfinite(run[:, 2]).any()
+                 else None}
+        if key in hbm_bytes:
+            gbs = hbm_bytes[key] / (med * 1e-6) / 1e9
+            entry.update(gbs=gbs, hbm_frac=gbs / peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
+        if key in flops:
+            tf = flops[key] / (med * 1e-6) / 1e12
+            entry.update(tflops_algorithmic=tf,
+                         tensor_frac=tf / peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
+        out[key] = entry
+    line = {"timeline": out, "workload": workload_desc(cfg, batch)["workload"], "steps": args.steps,
+            "warmup": args.warmup, "peaks": peak_kind,
+            "method": "GPU global timer in the traced library; L2 flushed before each step; the host reads "
+                      "the timeline after each merge, so the two merges do not overlap"}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
         return run_reference(args)
+    if args.timeline:
+        return run_timeline(args)
     return run_mpm(args)
 
 

@@ -335,6 +335,38 @@ MPM_API mpm_status mpm_get_device_status(void* workspace, int32_t* host_code, vo
  */
 MPM_API mpm_status mpm_selftest_wait_timeout(int32_t* device_status, uint32_t limit_us, void* stream);
 
+/*
+ * Device timeline of the merge, compose and gather kernels (the paper has no
+ * counterpart).  Only a library built with tracing (build(trace=True), which
+ * writes libmpm_trace.so) records it; the ordinary library returns
+ * MPM_ERR_UNSUPPORTED from both calls.
+ *
+ * For each kernel kind, the traced kernels keep three readings of the GPU
+ * global timer (ns):
+ *   [0] the earliest block start;
+ *   [1] the earliest moment a block passed its wait for the previous
+ *       kernel in the stream;
+ *   [2] the latest moment one of its warps finished.
+ * A kind that did not run since the last reset reads UINT64_MAX in [0] and
+ * [1] and 0 in [2].  Launches of the same kind since the reset are folded
+ * together, so reset between the launches you want to tell apart.
+ *
+ * mpm_trace_read copies MPM_TRACE_KINDS x 3 uint64 values into `out`, a
+ * host array.  It is synchronous: call it after the traced work finished.
+ * mpm_trace_reset is synchronous too.
+ */
+typedef enum {
+  MPM_TRACE_PREP = 0,
+  MPM_TRACE_AFFINITY = 1,
+  MPM_TRACE_MUTUAL = 2,
+  MPM_TRACE_PAIR_AVERAGE = 3,
+  MPM_TRACE_GATHER = 4,
+  MPM_TRACE_COMPOSE = 5,
+  MPM_TRACE_KINDS = 6
+} mpm_trace_kind;
+MPM_API mpm_status mpm_trace_read(uint64_t* out);
+MPM_API mpm_status mpm_trace_reset(void);
+
 #ifdef __cplusplus
 }
 #endif

@@ -16,6 +16,8 @@ from .mpm import (  # noqa: F401
     new_workspace,
     pad_batch,
     selftest_wait_timeout,
+    trace_read,
+    trace_reset,
     unmerge_gather,
     unpad_batch,
     workspace_size,

@@ -18,6 +18,10 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libmpm.so")
+# The same sources with the device timeline compiled in (-DMPM_TRACE); see
+# mpm_trace_read in include/mpm.h.  Used by `bench.py --timeline` only.
+BUILD_TRACE = os.path.join(PKG, "_build_trace")
+LIB_TRACE = os.path.join(PKG, "libmpm_trace.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-fvisibility=hidden",
                      "-I", os.path.join(ROOT, "include"), "-I", CSRC]
@@ -48,28 +52,30 @@ def _run(cmd: list) -> None:
         raise RuntimeError(f"command failed ({res.returncode}): {' '.join(cmd)}\n{res.stdout}\n{res.stderr}")
 
 
-def build(force: bool = False, extra_flags: list | None = None) -> str:
-    """Compiles and links libmpm.so if any source changed; returns its path."""
-    os.makedirs(BUILD, exist_ok=True)
+def build(force: bool = False, extra_flags: list | None = None, trace: bool = False) -> str:
+    """Compiles and links libmpm.so (libmpm_trace.so with trace=True) if any
+    source changed; returns its path."""
+    build_dir, lib_path = (BUILD_TRACE, LIB_TRACE) if trace else (BUILD, LIB)
+    os.makedirs(build_dir, exist_ok=True)
     srcs = sorted(glob.glob(os.path.join(CSRC, "*.cu")))
     headers = _headers()
-    flags = NVCC_FLAGS + list(extra_flags or [])
+    flags = NVCC_FLAGS + (["-DMPM_TRACE"] if trace else []) + list(extra_flags or [])
     jobs = []
     objs = []
     for src in srcs:
-        obj = os.path.join(BUILD, os.path.basename(src)[:-3] + ".o")
+        obj = os.path.join(build_dir, os.path.basename(src)[:-3] + ".o")
         objs.append(obj)
         if force or _stale(obj, [src] + headers):
             jobs.append([nvcc(), "-c", src, "-o", obj] + flags)
     if jobs:
         with concurrent.futures.ThreadPoolExecutor(max_workers=min(8, len(jobs))) as ex:
             list(ex.map(_run, jobs))
-    if force or jobs or _stale(LIB, objs):
-        tmp = LIB + ".tmp"
+    if force or jobs or _stale(lib_path, objs):
+        tmp = lib_path + ".tmp"
         _run([nvcc(), "-shared", "-o", tmp] + objs + ARCH +
              ["-cudart", "static", "-Xlinker", "--version-script=" + os.path.join(CSRC, "exports.map")])
-        os.replace(tmp, LIB)
-    return LIB
+        os.replace(tmp, lib_path)
+    return lib_path
 
 
 if __name__ == "__main__":

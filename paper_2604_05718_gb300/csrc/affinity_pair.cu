@@ -284,6 +284,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     affinity_pair_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constant__ CUtensorMap tmap_lo,
                          int batch, int dim, int64_t chunk, Workspace ws) {
   constexpr int kBK = TF32 ? TF_BK : BK;
+  MPM_TRACE_BEGIN(MPM_TRACE_AFFINITY);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024u - (ptx::smem_addr(smem_raw) & 1023u)) & 1023u);
   uint8_t* stages = smem;
@@ -333,6 +334,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   // Everything above touches no data of earlier kernels; from here on the
   // work plan, offsets and norms written by the prep kernel are read.
   wait_for_previous_grid();
+  MPM_TRACE_WAITED();
   const bool staged = batch <= kMaxStagedImages;
   if (staged) {
     for (int e = threadIdx.x; e <= batch; e += THREADS) {
@@ -569,6 +571,10 @@ PFN_cuTensorMapEncodeTiled_v12000 encoder() {
 }
 
 }  // namespace
+
+#ifdef MPM_TRACE
+cudaError_t trace_copy_pair(unsigned long long* out, bool reset) { return trace_table(out, reset); }
+#endif
 
 AffinityTile pair_tile() { return {TILE, TILE, AffinityTile::kUpperSquare}; }
 

@@ -9,6 +9,7 @@
 #include <utility>
 
 #include "launch.h"
+#include "mpm.h"
 
 namespace mpm {
 
@@ -49,6 +50,51 @@ inline int resident_per_sm(void (*kernel)(Params...), int threads, int cap) {
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kernel, threads, 0) != cudaSuccess || n < 1) return cap;
   return n < cap ? n : cap;
 }
+
+// ---------------------------------------------------------------------------
+// Device timeline (libmpm_trace.so only; see mpm_trace_read in mpm.h).  Each
+// translation unit with traced kernels keeps its own table, which
+// trace_copy_<unit> reads or resets from the host.
+// ---------------------------------------------------------------------------
+#ifdef MPM_TRACE
+static __device__ unsigned long long g_trace[MPM_TRACE_KINDS][3];
+__device__ __forceinline__ unsigned long long trace_now() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+struct TraceScope {
+  int kind;
+  __device__ explicit TraceScope(int k) : kind(k) {
+    if (threadIdx.x == 0) atomicMin(&g_trace[kind][0], trace_now());
+  }
+  __device__ void waited() const {
+    if (threadIdx.x == 0) atomicMin(&g_trace[kind][1], trace_now());
+  }
+  __device__ ~TraceScope() {
+    if ((threadIdx.x & 31) == 0) atomicMax(&g_trace[kind][2], trace_now());
+  }
+};
+// Reads (reset == false) or resets this translation unit's table.
+static inline cudaError_t trace_table(unsigned long long* out, bool reset) {
+  if (!reset) return cudaMemcpyFromSymbol(out, g_trace, sizeof(g_trace));
+  unsigned long long v[MPM_TRACE_KINDS][3];
+  for (int k = 0; k < MPM_TRACE_KINDS; ++k) {
+    v[k][0] = v[k][1] = ~0ull;
+    v[k][2] = 0ull;
+  }
+  return cudaMemcpyToSymbol(g_trace, v, sizeof(v));
+}
+#define MPM_TRACE_BEGIN(kind) const ::mpm::TraceScope mpm_trace_scope_(kind)
+#define MPM_TRACE_WAITED() mpm_trace_scope_.waited()
+#else
+#define MPM_TRACE_BEGIN(kind) \
+  do {                         \
+  } while (0)
+#define MPM_TRACE_WAITED() \
+  do {                     \
+  } while (0)
+#endif
 
 // First error wins; `st` may be null (not reported).
 __device__ __forceinline__ void report(int32_t* st, int32_t code, int32_t detail) {

@@ -44,7 +44,9 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(const uint8_t* __restric
                                                         int batch, int64_t rows, int row_bytes,
                                                         bool bf16, AffinityTile tile,
                                                         Workspace ws) {
+  MPM_TRACE_BEGIN(MPM_TRACE_PREP);
   wait_for_previous_grid();
+  MPM_TRACE_WAITED();
   // The affinity kernel that follows only sets up barriers and tensor memory
   // before it waits for this grid, so it may take SMs as this grid drains.
   // (The other kernels do not trigger early: blocks of a dependent grid
@@ -168,7 +170,9 @@ constexpr int kScanThreads = 1024;
 __global__ void __launch_bounds__(kScanThreads) mutual_compact_kernel(int batch, int64_t chunk, Workspace ws,
                                                                       int32_t* __restrict__ out_map,
                                                                       int64_t* __restrict__ out_offsets) {
+  MPM_TRACE_BEGIN(MPM_TRACE_MUTUAL);
   wait_for_previous_grid();
+  MPM_TRACE_WAITED();
   __shared__ int32_t sh[32];
   __shared__ int64_t sh64[32];
   __shared__ int is_last;
@@ -233,7 +237,9 @@ __global__ void __launch_bounds__(kThreads) pair_average_kernel(const uint8_t* _
                                                                 int batch, int64_t rows, int row_bytes,
                                                                 bool bf16, Workspace ws,
                                                                 const int64_t* __restrict__ out_offsets) {
+  MPM_TRACE_BEGIN(MPM_TRACE_PAIR_AVERAGE);
   wait_for_previous_grid();
+  MPM_TRACE_WAITED();
   const int lane = threadIdx.x & 31;
   const int64_t warp = (static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x) >> 5;
   const int64_t nwarps = (static_cast<int64_t>(gridDim.x) * kThreads) >> 5;
@@ -310,7 +316,9 @@ __global__ void compose_kernel(const int32_t* map1, const int64_t* __restrict__ 
                                int64_t rows0, const int32_t* __restrict__ map2,
                                const int64_t* __restrict__ off1, int64_t rows1, int batch,
                                int32_t* out, int32_t* status) {
+  MPM_TRACE_BEGIN(MPM_TRACE_COMPOSE);
   wait_for_previous_grid();
+  MPM_TRACE_WAITED();
   const int64_t used = clamp64(off0[batch], 0, rows0);
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   for (int64_t p = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; p < used; p += stride) {
@@ -347,7 +355,9 @@ __global__ void __launch_bounds__(kThreads) gather_kernel(const uint8_t* __restr
                                                           const int64_t* __restrict__ off1, int64_t rows1,
                                                           int32_t* out_map, int batch, int row_bytes,
                                                           uint8_t* __restrict__ out, int32_t* status) {
+  MPM_TRACE_BEGIN(MPM_TRACE_GATHER);
   wait_for_previous_grid();
+  MPM_TRACE_WAITED();
   const int lane = threadIdx.x & 31;
   const int64_t warp = (static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x) >> 5;
   const int64_t nwarps = (static_cast<int64_t>(gridDim.x) * kThreads) >> 5;
@@ -407,6 +417,10 @@ __global__ void __launch_bounds__(kThreads) gather_kernel(const uint8_t* __restr
 int grid_for(int num_sms, int per_sm) { return (num_sms > 0 ? num_sms : 1) * per_sm; }
 
 }  // namespace
+
+#ifdef MPM_TRACE
+cudaError_t trace_copy_hbm(unsigned long long* out, bool reset) { return trace_table(out, reset); }
+#endif
 
 cudaError_t launch_prep(const void* tokens, const int64_t* offsets, int batch, int64_t rows, int dim,
                         bool bf16, AffinityTile tile, const Workspace& ws, int num_sms,

@@ -94,6 +94,13 @@ cudaError_t launch_compose_gather(const void* merged, const int64_t* moff, int64
                                   bool bf16, void* out, int32_t* out_map, int32_t* status, int num_sms,
                                   cudaStream_t stream);
 
+#ifdef MPM_TRACE
+// Device timeline tables of kernels_hbm.cu and affinity_pair.cu (MPM_TRACE
+// builds): copy out (reset == false) or reset.
+cudaError_t trace_copy_hbm(unsigned long long* out, bool reset);
+cudaError_t trace_copy_pair(unsigned long long* out, bool reset);
+#endif
+
 // Padded batch [batch, max_len, dim] + key mask + N_b statistics, and its
 // inverse (kernels_pad.cu).
 cudaError_t launch_pad(const void* tokens, const int64_t* offsets, int batch, int64_t rows, int64_t max_len,

@@ -411,6 +411,36 @@ mpm_status mpm_unpad_batch(const void* padded, int32_t batch, int64_t max_len, i
                                        device_status, sms, static_cast<cudaStream_t>(stream)));
 }
 
+mpm_status mpm_trace_read(uint64_t* out) {
+#ifdef MPM_TRACE
+  if (out == nullptr) return MPM_ERR_INVALID_ARG;
+  unsigned long long a[MPM_TRACE_KINDS][3], b[MPM_TRACE_KINDS][3];
+  if (cudaDeviceSynchronize() != cudaSuccess || mpm::trace_copy_hbm(&a[0][0], false) != cudaSuccess ||
+      mpm::trace_copy_pair(&b[0][0], false) != cudaSuccess)
+    return MPM_ERR_CUDA;
+  for (int k = 0; k < MPM_TRACE_KINDS; ++k) {
+    out[3 * k + 0] = a[k][0] < b[k][0] ? a[k][0] : b[k][0];
+    out[3 * k + 1] = a[k][1] < b[k][1] ? a[k][1] : b[k][1];
+    out[3 * k + 2] = a[k][2] > b[k][2] ? a[k][2] : b[k][2];
+  }
+  return MPM_OK;
+#else
+  (void)out;
+  return MPM_ERR_UNSUPPORTED;
+#endif
+}
+
+mpm_status mpm_trace_reset(void) {
+#ifdef MPM_TRACE
+  if (cudaDeviceSynchronize() != cudaSuccess || mpm::trace_copy_hbm(nullptr, true) != cudaSuccess ||
+      mpm::trace_copy_pair(nullptr, true) != cudaSuccess)
+    return MPM_ERR_CUDA;
+  return MPM_OK;
+#else
+  return MPM_ERR_UNSUPPORTED;
+#endif
+}
+
 mpm_status mpm_get_device_status(void* workspace, int32_t* host_code, void* stream) {
   if (workspace == nullptr || host_code == nullptr) return MPM_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);

@@ -18,6 +18,9 @@ import os
 import torch
 
 LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libmpm.so")
+# The same library with the device timeline compiled in (build(trace=True)).
+TRACE_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libmpm_trace.so")
+TRACE_KINDS = ("prep", "affinity", "mutual_scan", "pair_average", "gather", "compose")
 
 MPM_F32, MPM_BF16 = 0, 1
 ALGOS = {"auto": 0, "simt": 1, "tcgen05": 2, "tcgen05_sym": 3, "tcgen05_pair": 4}
@@ -64,6 +67,8 @@ def _declare(lib: ctypes.CDLL) -> None:
                                                          P, SZ, P]),
         "mpm_unpad_batch": (ctypes.c_int, [P, I32, I64, I32, ctypes.c_int, P, I64, P, P, P]),
         "mpm_selftest_wait_timeout": (ctypes.c_int, [P, ctypes.c_uint32, P]),
+        "mpm_trace_read": (ctypes.c_int, [P]),
+        "mpm_trace_reset": (ctypes.c_int, []),
     }
     for name, (res, args) in sigs.items():
         fn = getattr(lib, name)
@@ -363,3 +368,25 @@ def selftest_wait_timeout(limit_us: int, device=None) -> torch.Tensor:
         code = library().mpm_selftest_wait_timeout(_ptr(status), int(limit_us), _stream(dev))
     _check("mpm_selftest_wait_timeout", code)
     return status
+
+
+def trace_reset() -> None:
+    """Clears the device timeline (libmpm_trace.so only; synchronous)."""
+    _check("mpm_trace_reset", library().mpm_trace_reset())
+
+
+def trace_read() -> dict:
+    """Device timeline since the last reset (libmpm_trace.so only;
+    synchronous): for each kernel kind that ran, (first block start, first
+    block past its wait for the previous kernel, last warp end) in ns of the
+    GPU global timer."""
+    import numpy as np
+
+    out = np.zeros(3 * len(TRACE_KINDS), dtype=np.uint64)
+    _check("mpm_trace_read", library().mpm_trace_read(out.ctypes.data))
+    res = {}
+    for k, name in enumerate(TRACE_KINDS):
+        start, waited, end = (int(v) for v in out[3 * k:3 * k + 3])
+        if end != 0:
+            res[name] = (start, waited, end)
+    return res
