@@ -72,3 +72,17 @@ def test_traced_library_timeline_and_results():
     assert off1.cpu().tolist() == got["off1"]
     assert m1[:b.rows].cpu().tolist() == got["map1"]
     np.testing.assert_array_equal(x1[:int(off1[-1])].float().cpu().numpy().round(6)[:50], np.array(got["x1"]))
+
+
+def test_bench_timeline_mode():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    res = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--timeline", "--steps", "2",
+                          "--warmup", "1"], capture_output=True, text=True, cwd=ROOT, timeout=900)
+    assert res.returncode == 0, res.stderr[-2000:]
+    d = json.loads(res.stdout.strip().splitlines()[-1])
+    tl = d["timeline"]
+    for key in ("prep_1", "affinity_1", "mutual_scan_1", "pair_average_1", "prep_2", "affinity_2",
+                "mutual_scan_2", "pair_average_2", "gather"):
+        assert tl[key]["us_after_wait"] > 0, key
+    assert tl["affinity_1"]["tflops_algorithmic"] > 0 and tl["pair_average_1"]["gbs"] > 0
