@@ -64,6 +64,8 @@ def parse_args():
     p.add_argument("--no-chunked", action="store_true", help="skip the chunked-similarity measurement")
     p.add_argument("--no-padded", action="store_true", help="skip the padded-batch measurement")
     p.add_argument("--no-fp32", action="store_true", help="skip the fp32 nearest-neighbour measurement")
+    p.add_argument("--no-timeline", action="store_true",
+                   help="skip the in-step device timeline (traced library, child process) of the default run")
     p.add_argument("--timeline", action="store_true",
                    help="instead of the benchmark, print each kernel's in-step duration from the device "
                         "timeline of the traced library (libmpm_trace.so); one GPU")
@@ -703,6 +705,13 @@ def run_mpm(args):
                "pipeline": "3 streams: copy in of step k+1 and copy out of step k-1 overlap step k; "
                            "timed from the first copy in to the last copy out"}
 
+    # The same step on the traced library, in a child process: each kernel's
+    # duration inside the step (device timer), next to the CUDA-event figures
+    # above, which add launch latency.  roofline.achieved stays the event one.
+    in_step = None
+    if rank == 0 and world == 1 and not args.no_timeline:
+        in_step = in_step_timeline(args.workload)
+
     if world > 1:
         dist.barrier()
     if rank == 0:
@@ -720,6 +729,7 @@ def run_mpm(args):
             "fp32_nearest_neighbours": fp32,
             "kernels_us": kern,
             "ms_per_step_with_kernel_events": ms_with_kernel_events,
+            "in_step": in_step,
             "cpu_baseline": cpu_base,
             "e2e": e2e,
             "clocks": clk,
@@ -735,6 +745,33 @@ def run_mpm(args):
 # ---------------------------------------------------------------------------
 # Device timeline of the step (traced library)
 # ---------------------------------------------------------------------------
+def in_step_timeline(workload):
+    """Runs `bench.py --timeline` for `workload` in a child process (one MPM
+    library per process) and condenses its line; None if it fails."""
+    import subprocess
+
+    cmd = [sys.executable, os.path.abspath(__file__), "--timeline", "--workload", workload, "--steps", "10",
+           "--warmup", "3"]
+    try:
+        res = subprocess.run(cmd, capture_output=True, text=True, timeout=600, cwd=ROOT)
+        tl = json.loads(res.stdout.strip().splitlines()[-1])["timeline"]
+    except (subprocess.SubprocessError, OSError, ValueError, IndexError, KeyError):
+        return None
+    aff = [k for k in ("affinity_1", "affinity_2") if k in tl]
+    us = sum(tl[k]["us_after_wait"] for k in aff)
+    tflop = sum(tl[k]["tflops_algorithmic"] * tl[k]["us_after_wait"] * 1e-6 for k in aff)
+    peaks, _ = load_peaks()
+    tf = tflop / (us * 1e-6)
+    return {
+        "source": "python bench.py --timeline --steps 10 --warmup 3 (traced library, GPU global timer, medians)",
+        "kernels_us": {k: v["us_after_wait"] for k, v in tl.items()},
+        "affinity_tflops_algorithmic": tf,
+        "affinity_frac_of_sustained_bf16": tf / peaks.get("bf16_tflops_sustained",
+                                                            FALLBACK_PEAKS["bf16_tflops_sustained"]),
+        "hbm_gbs": {k: v["gbs"] for k, v in tl.items() if "gbs" in v},
+    }
+
+
 def run_timeline(args):
     """The benchmark step with the device timeline of libmpm_trace.so: for
     every kernel, the time from the moment its blocks passed their wait for

@@ -38,3 +38,7 @@ def test_gpu_arm_prints_one_contract_line():
     c = d["clocks"]
     assert {"sm_mhz", "sm_max_mhz", "reasons"} <= set(c)
     assert d["gpu_launches"] == 9 * d["steps"]   # four kernels per merge, two merges, one compose + gather
+    # The in-step timeline of the traced library, beside the event figures.
+    ins = d["in_step"]
+    assert ins is not None and ins["affinity_tflops_algorithmic"] > 0
+    assert set(ins["kernels_us"]) >= {"prep_1", "affinity_1", "mutual_scan_1", "pair_average_1", "gather"}
