@@ -167,6 +167,33 @@ def test_many_tiny_images(mpm, algo):
     merge_parity(mpm, batch, "16000 tiny images", algo=algo)
 
 
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_merge_is_bitwise_deterministic(mpm, dtype):
+    # Candidates from many tiles meet in 64-bit atomicMax on packed (score,
+    # lowest index) keys, so the order in which the SM pairs finish cannot
+    # change a result: three merges (two workspaces, two streams) agree bit
+    # for bit.
+    batch = make_custom([1024] * 24 + [700, 513, 1, 0], 768 if dtype == "bf16" else 256, dtype, seed=47)
+    x = batch.tokens.to(DEV)
+    off = torch.from_numpy(batch.offsets).to(DEV)
+    runs = []
+    side = torch.cuda.Stream()
+    for k in range(3):
+        ws = mpm.new_workspace(x.shape[0], batch.batch, x.shape[1], x.dtype, DEV)
+        stream = side if k == 2 else torch.cuda.current_stream()
+        stream.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(stream):
+            out, out_off, rmap = mpm.merge(x, off, workspace=ws)
+        torch.cuda.synchronize()
+        t = int(out_off[-1])
+        runs.append((out[:t].cpu(), out_off.cpu(), rmap[:batch.rows].cpu()))
+    for other in runs[1:]:
+        assert torch.equal(runs[0][1], other[1])
+        assert torch.equal(runs[0][2], other[2])
+        assert torch.equal(runs[0][0].view(torch.int16 if dtype == "bf16" else torch.int32),
+                           other[0].view(torch.int16 if dtype == "bf16" else torch.int32))
+
+
 def test_tcgen05_and_simt_agree(mpm):
     batch = make_custom([1000, 513, 64, 2300], 384, "bf16", seed=9)
     runs = {algo: run_merge(mpm, batch.tokens, batch.offsets, algo)
