@@ -125,3 +125,48 @@ def exact_maximisers(x: list, i: int) -> set:
         if _cmp_ratio(dj, qj, db, qb) == 0:
             out.add(j)
     return out
+
+
+def _cos_decimal(x: list, i: int, j: int):
+    """cos(x_i, x_j) to 50 significant digits; 0 when either token is zero."""
+    from decimal import Decimal, localcontext
+
+    qi, qj = _dot(x[i], x[i]), _dot(x[j], x[j])
+    if qi == 0 or qj == 0:
+        return Decimal(0)
+    with localcontext() as ctx:
+        ctx.prec = 50
+        return Decimal(_dot(x[i], x[j])) / (Decimal(qi) * Decimal(qj)).sqrt()
+
+
+def exact_row_diagnostics(x: list, i: int):
+    """Best and second-best cosine of row i over j != i (Section 3.2's b(i) and runner-up).
+
+    Candidates are ordered by the exact comparator (no rounding decides the
+    order); the two values are then evaluated to 50 digits.  Returns
+    (top1, top2, tied): top1/top2 are Decimals or None for "no candidate"
+    (-inf), and tied is True when the two best candidates have exactly equal
+    cosines (gap exactly 0).
+    """
+    from functools import cmp_to_key
+
+    n = len(x)
+    cands = [j for j in range(n) if j != i]
+    if not cands:
+        return None, None, False
+    q = [_dot(v, v) for v in x]
+
+    def ratio(j):
+        if q[i] == 0 or q[j] == 0:
+            return 0, 1
+        return _dot(x[i], x[j]), q[j]
+
+    def cmp(a, b):  # descending by exact cosine
+        return -_cmp_ratio(*ratio(a), *ratio(b))
+
+    order = sorted(cands, key=cmp_to_key(cmp))
+    top1 = _cos_decimal(x, i, order[0])
+    if len(order) == 1:
+        return top1, None, False
+    tied = cmp(order[0], order[1]) == 0
+    return top1, _cos_decimal(x, i, order[1]), tied

@@ -18,7 +18,8 @@ import torch
 
 import oracle
 from oracle import mpm_oracle
-from exact_mpm import exact_maximisers, exact_merge, exact_nearest, exact_top_gap_positive
+from exact_mpm import (exact_maximisers, exact_merge, exact_nearest, exact_row_diagnostics,
+                       exact_top_gap_positive)
 from golden_io import load_hand_examples
 from workloads import make_custom
 
@@ -37,6 +38,17 @@ def check_hand_example(ex) -> None:
     np.testing.assert_allclose(res.x_out, means, rtol=0, atol=1e-15, err_msg=ex.name)
     if ex.x_out is not None:
         np.testing.assert_allclose(res.x_out, ex.x_out, rtol=0, atol=1e-15, err_msg=ex.name)
+    check_hand_diagnostics(ex, res.nn)
+
+
+def check_hand_diagnostics(ex, nn) -> None:
+    """Best / second-best cosine and the near-tie flag against the hand values."""
+    if ex.top1 is not None:
+        np.testing.assert_allclose(nn.top1, ex.top1, rtol=0, atol=1e-12, err_msg=ex.name + " top1")
+    if ex.top2 is not None:
+        np.testing.assert_allclose(nn.top2, ex.top2, rtol=0, atol=1e-12, err_msg=ex.name + " top2")
+    if ex.near_tie is not None:
+        assert nn.near_tie.astype(int).tolist() == ex.near_tie, ex.name + " near_tie"
 
 
 @pytest.mark.parametrize("ex", load_hand_examples(), ids=lambda e: e.name)
@@ -113,6 +125,100 @@ def test_exact_bruteforce_duplicate_ties():
             assert not any(xl[k] == xl[j] for k in range(j) if k != i), (xl, i)
             checked += 1
     assert checked > 1000
+
+
+# ---------------------------------------------------------------------------
+# Near-tie diagnostics: the runner-up cosine and the 1e-4 gap rule
+# ---------------------------------------------------------------------------
+def check_exact_diagnostics(seed_count: int = 300, seed: int = 20261202) -> tuple:
+    """top1 / top2 / near_tie against exact arithmetic on tiny integer tokens.
+
+    Small entries give many exact ties (gap 0: near-tie); wide entries give
+    gaps of every size.  A row whose exact gap lies within 1e-9 of the 1e-4
+    threshold is not judged (fp64 may round either way there).
+    Returns (decisive rows, near-tie rows without an exact tie, exact ties).
+    """
+    rng = np.random.default_rng(seed)
+    counts = [0, 0, 0]
+    for k in range(seed_count):
+        n = int(rng.integers(1, 9))
+        d = int(rng.integers(1, 6))
+        if k % 3 == 2:
+            # Near-parallel tokens (a, u, v) with a in [100, 400] and small
+            # integer offsets: cosines near 1 whose differences span 1e-6..1e-2.
+            n, d = int(rng.integers(3, 8)), 3
+            x = np.concatenate([rng.integers(100, 401, size=(n, 1)),
+                                rng.integers(-12, 13, size=(n, 2))], axis=1)
+        else:
+            hi = 3 if k % 3 == 0 else 60
+            x = _random_int_tokens(rng, n, d, -hi, hi)
+        xl = x.tolist()
+        nn = mpm_oracle.nearest_neighbours(x.astype(np.float64))
+        near = nn.near_tie
+        for i in range(n):
+            top1, top2, tied = exact_row_diagnostics(xl, i)
+            if top1 is None:
+                assert nn.top1[i] == -np.inf and nn.top2[i] == -np.inf and near[i], (xl, i)
+                continue
+            assert abs(nn.top1[i] - float(top1)) <= 1e-12, (xl, i)
+            if top2 is None:
+                assert nn.top2[i] == -np.inf and not near[i], (xl, i)
+                counts[0] += 1
+                continue
+            assert abs(nn.top2[i] - float(top2)) <= 1e-12, (xl, i)
+            if tied:
+                assert near[i], (xl, i)
+                counts[2] += 1
+                continue
+            gap = float(top1 - top2)
+            assert gap > 0, (xl, i)
+            if abs(gap - oracle.NEAR_TIE_GAP) <= 1e-9:
+                continue
+            assert bool(near[i]) == (gap < oracle.NEAR_TIE_GAP), (xl, i, gap)
+            counts[0 if gap > oracle.NEAR_TIE_GAP else 1] += 1
+    return tuple(counts)
+
+
+def test_exact_bruteforce_near_tie_diagnostics():
+    decisive, near_untied, ties = check_exact_diagnostics()
+    assert decisive > 500 and ties > 50 and near_untied > 50, (decisive, near_untied, ties)
+
+
+def check_near_tie_threshold() -> None:
+    """R14: a gap of exactly 1e-4 is near-tie ("exceeds" is strict).
+
+    The affinity rows are written out: row 0 has best 1e-4 and second 0
+    (gap == 1e-4 in fp64), row 1 best just above 1e-4 (gap > 1e-4), row 2
+    two equal candidates (gap 0).
+    """
+    above = np.nextafter(1e-4, 1.0)
+    s = np.array([[-np.inf, 1e-4, 0.0],
+                  [above, -np.inf, 0.0],
+                  [0.25, 0.25, -np.inf]])
+    nn = mpm_oracle.nearest_neighbours(np.eye(3), affinity=s)
+    assert nn.b.tolist() == [1, 0, 0]
+    assert nn.top1.tolist() == [1e-4, above, 0.25] and nn.top2.tolist() == [0.0, 0.0, 0.25]
+    assert nn.gap[0] == oracle.NEAR_TIE_GAP
+    assert nn.near_tie.tolist() == [True, False, True]
+
+
+def test_near_tie_threshold_is_strict():
+    check_near_tie_threshold()
+
+
+def test_chunked_runner_up_stays_in_the_chunk():
+    """Under chunking the runner-up is sought inside the row's chunk only (Section 5 reading).
+
+    Chunks of 2: each row has a single candidate, so top2 is -inf and no row
+    is near-tie, although the full image would tie (identical tokens).
+    """
+    x = np.tile(np.array([[1.0, 2.0, -1.0]]), (5, 1))
+    full = mpm_oracle.nearest_neighbours(x)
+    assert full.near_tie.all()
+    nn = mpm_oracle.nearest_neighbours(x, chunk=2)
+    assert nn.b.tolist() == [1, 0, 3, 2, -1]
+    np.testing.assert_allclose(nn.top1[:4], 1.0, atol=1e-15)
+    assert np.all(nn.top2 == -np.inf) and nn.near_tie.tolist() == [False] * 4 + [True]
 
 
 # ---------------------------------------------------------------------------
@@ -300,6 +406,13 @@ def test_chunked_exact_bruteforce_tiny():
                 j = int(got.nn.b[c0 + i])
                 assert c0 <= j < c0 + len(part), (part, i, j)
                 assert j - c0 in exact_maximisers(part, i), (part, i, j)
+                top1, top2, tied = exact_row_diagnostics(part, i)
+                assert abs(got.nn.top1[c0 + i] - float(top1)) <= 1e-12, (part, i)
+                if top2 is None:
+                    assert got.nn.top2[c0 + i] == -np.inf, (part, i)
+                else:
+                    assert abs(got.nn.top2[c0 + i] - float(top2)) <= 1e-12, (part, i)
+                    assert not tied or got.nn.near_tie[c0 + i], (part, i)
                 checked += 1
     assert checked > 500
 
@@ -386,6 +499,8 @@ def _all_pins_pass() -> bool:
         for ex in load_hand_examples():
             check_hand_example(ex)
         check_exact_bruteforce(120)
+        check_exact_diagnostics(120)
+        check_near_tie_threshold()
         test_duplicate_pairs_far_apart()
         rng = np.random.default_rng(0)
         check_invariants(rng.standard_normal((50, 6)))
@@ -480,19 +595,65 @@ def _average_first(x, r, n_out):
     return out
 
 
+def _affinity_for(x, affinity, chunk):
+    return mpm_oracle.cosine_affinity(x, chunk) if affinity is None else affinity
+
+
+def _nn_top2_drops_ties(x, affinity=None, chunk=None):
+    # Runner-up taken among the candidates strictly below the best: an exact
+    # tie then looks like a clear win.
+    nn = _orig_nn(x, affinity, chunk)
+    if nn.b.shape[0] > 2:
+        s = _affinity_for(x, affinity, chunk)
+        nn.top2 = np.where(s >= nn.top1[:, None], -np.inf, s).max(axis=1)
+    return nn
+
+
+def _nn_top2_row_min(x, affinity=None, chunk=None):
+    # Runner-up replaced by the worst candidate.
+    nn = _orig_nn(x, affinity, chunk)
+    if nn.b.shape[0] > 2:
+        s = _affinity_for(x, affinity, chunk)
+        nn.top2 = np.where(np.isneginf(s), np.inf, s).min(axis=1)
+    return nn
+
+
+def _nn_top2_keeps_self(x, affinity=None, chunk=None):
+    # Runner-up searched over an affinity whose diagonal was never masked.
+    nn = _orig_nn(x, affinity, chunk)
+    n = nn.b.shape[0]
+    if n > 2:
+        xt = mpm_oracle.normalise_rows(x)
+        s = xt @ xt.T
+        s[np.arange(n), nn.b] = -np.inf
+        nn.top2 = s.max(axis=1)
+    return nn
+
+
 _orig_nn = mpm_oracle.nearest_neighbours
 _orig_compact = mpm_oracle.compact_map
+_N = mpm_oracle.Neighbours
 
 MUTATIONS = {
-    "tie_to_highest_j": ("nearest_neighbours", _nn_highest_tie),
-    "no_diagonal_mask": ("nearest_neighbours", _nn_no_mask),
-    "argmin_instead_of_argmax": ("nearest_neighbours", _nn_argmin),
-    "dot_not_cosine": ("nearest_neighbours", _nn_unnormalised),
-    "pairs_not_mutual": ("mutual_partners", _partners_not_mutual),
-    "upper_index_representative": ("compact_map", _compact_upper_rep),
-    "one_based_ids": ("compact_map", _compact_one_based),
-    "sum_not_mean": ("cluster_average", _average_sum),
-    "keep_first_member": ("cluster_average", _average_first),
+    "tie_to_highest_j": (mpm_oracle, "nearest_neighbours", _nn_highest_tie),
+    "no_diagonal_mask": (mpm_oracle, "nearest_neighbours", _nn_no_mask),
+    "argmin_instead_of_argmax": (mpm_oracle, "nearest_neighbours", _nn_argmin),
+    "dot_not_cosine": (mpm_oracle, "nearest_neighbours", _nn_unnormalised),
+    "pairs_not_mutual": (mpm_oracle, "mutual_partners", _partners_not_mutual),
+    "upper_index_representative": (mpm_oracle, "compact_map", _compact_upper_rep),
+    "one_based_ids": (mpm_oracle, "compact_map", _compact_one_based),
+    "sum_not_mean": (mpm_oracle, "cluster_average", _average_sum),
+    "keep_first_member": (mpm_oracle, "cluster_average", _average_first),
+    # Near-tie diagnostics (Section 3.2's b(i) runner-up and the 1e-4 gap rule).
+    "gap_always_zero": (_N, "gap", property(lambda self: np.zeros_like(self.top1))),
+    "gap_sign_flipped": (_N, "gap", property(lambda self: self.top2 - self.top1)),
+    "near_tie_at_or_above_threshold": (
+        _N, "near_tie", property(lambda self: ~(self.gap >= mpm_oracle.NEAR_TIE_GAP))),
+    "near_tie_ignores_undefined_gap": (
+        _N, "near_tie", property(lambda self: self.gap <= mpm_oracle.NEAR_TIE_GAP)),
+    "top2_drops_ties_of_top1": (mpm_oracle, "nearest_neighbours", _nn_top2_drops_ties),
+    "top2_is_row_minimum": (mpm_oracle, "nearest_neighbours", _nn_top2_row_min),
+    "top2_sees_the_diagonal": (mpm_oracle, "nearest_neighbours", _nn_top2_keeps_self),
 }
 
 
@@ -502,8 +663,8 @@ def test_pins_pass_on_the_oracle():
 
 @pytest.mark.parametrize("name", sorted(MUTATIONS))
 def test_pins_catch_planted_mistake(name, monkeypatch):
-    attr, fn = MUTATIONS[name]
-    monkeypatch.setattr(mpm_oracle, attr, fn)
+    owner, attr, value = MUTATIONS[name]
+    monkeypatch.setattr(owner, attr, value)
     assert not _all_pins_pass(), f"planted mistake {name} went unnoticed"
 
 
