@@ -16,3 +16,13 @@ for p in (ROOT, TESTS):
 
 def pytest_configure(config):
     config.addinivalue_line("markers", "gpu: needs a CUDA GPU and the compiled MPM library")
+
+
+def pytest_terminal_summary(terminalreporter, exitstatus, config):
+    """Print the parity records of the full-size workload tests, if any ran."""
+    parity = sys.modules.get("parity")
+    lines = getattr(parity, "SUMMARY_LINES", None) if parity else None
+    if lines:
+        terminalreporter.section("MPM parity on the full workloads")
+        for line in lines:
+            terminalreporter.write_line(line)

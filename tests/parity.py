@@ -31,6 +31,10 @@ import oracle
 
 TOL = {"f32": 1e-5, "bf16": 2e-3}
 
+# One machine-readable line per checked workload, printed in pytest's
+# terminal summary by tests/conftest.py.
+SUMMARY_LINES: list = []
+
 
 def to_f64(t: torch.Tensor) -> np.ndarray:
     return t.detach().cpu().double().numpy()
