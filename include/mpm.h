@@ -154,21 +154,41 @@ MPM_API mpm_status mpm_merge_timed(const void* tokens, const int64_t* offsets, i
  * the process exits.
  *  - Limit: it returns MPM_ERR_WORKSPACE when
  *    mpm_merge_workspace_size(rows, batch, dim, dtype) exceeds
- *    MPM_NO_ALLOC_SCRATCH_BYTES (8 MiB: about 400,000 rows at up to 1024
- *    images), and allocates nothing in any case.
- *  - The first call on each device looks up the array's device address
- *    (cudaGetSymbolAddress, which can load the module); make that first call
- *    before any stream capture on that device.
+ *    MPM_NO_ALLOC_SCRATCH_BYTES (8 MiB), and allocates nothing in any case.
+ *    The workspace takes about 20 bytes per row for bf16 tokens, so 8 MiB
+ *    holds about 400,000 rows; for fp32 tokens it also holds the two tf32
+ *    split copies of the tokens, 20 + 8 * dim bytes per row: about 5,400
+ *    rows at dim 192 and 1,360 rows at dim 768.  (Plus 20 bytes per image
+ *    and up to 256 bytes of alignment per region either way.)
+ *  - Set-up: the array's device address is looked up (cudaGetSymbolAddress,
+ *    which can load the module) once per device context, by the first call
+ *    on that device; make that first call before any stream capture on the
+ *    device.  It is looked up again only after the device's context changed
+ *    (a cudaDeviceReset between calls).
  *  - All calls on a device share the one array: calls that overlap on the
  *    GPU (different streams or host threads) race and must be serialised by
  *    the caller.  The array keeps the last call's contents; each call clears
- *    the part that must start at zero.  The device status word lives in the
- *    shared array and is not readable through mpm_get_device_status.
+ *    the part that must start at zero, including the device status word.
+ *  - Device-detected errors (offsets that are not monotone, a bounded wait
+ *    that ran out) go to the status word inside the shared array: read them
+ *    with mpm_no_alloc_get_device_status, after this call and before the
+ *    next one on the device.
  */
 #define MPM_NO_ALLOC_SCRATCH_BYTES (8u << 20)
 MPM_API mpm_status mpm_merge_no_alloc(const void* tokens, const int64_t* offsets, int32_t batch,
                                       int64_t rows, int32_t dim, mpm_dtype dtype, void* out_tokens,
                                       int64_t* out_offsets, int32_t* out_map, void* stream);
+
+/*
+ * The status word of the no-alloc scratch array on the current device, for
+ * callers of mpm_merge_no_alloc (no counterpart in the paper).  Like
+ * mpm_get_device_status: copies the first device-detected error of the last
+ * mpm_merge_no_alloc call on this device into *host_code (0 = none;
+ * otherwise MPM_ERR_DEVICE_CHECK or MPM_ERR_DEVICE_TIMEOUT), synchronising
+ * `stream`, then clears the word.  Allocates nothing.
+ * Errors: MPM_ERR_INVALID_ARG (host_code NULL), MPM_ERR_CUDA.
+ */
+MPM_API mpm_status mpm_no_alloc_get_device_status(int32_t* host_code, void* stream);
 
 /*
  * Chunked similarity: mpm_merge with each token's nearest neighbour sought

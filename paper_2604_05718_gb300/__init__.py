@@ -12,8 +12,10 @@ from .mpm import (  # noqa: F401
     device_status,
     library,
     merge,
+    merge_no_alloc,
     nearest_neighbors,
     new_workspace,
+    no_alloc_device_status,
     pad_batch,
     selftest_wait_timeout,
     trace_read,

@@ -12,16 +12,19 @@
 //
 // The array is a file-scope __device__ variable: every GPU that loads the
 // library holds one copy of it until the process exits.  Host code cannot
-// use its name as a device address, so the first call on each device looks
-// the address up with cudaGetSymbolAddress (with that device current) and
-// caches it.  That first call can load the module and must therefore come
-// before any stream capture on that device.
+// use its name as a device address.  The set-up looks the address up with
+// cudaGetSymbolAddress, with the device current, once per device context:
+// the first call on a device does it (it can load the module, so that first
+// call must come before any stream capture on the device), and it is done
+// again only if the device's context changed since (a cudaDeviceReset
+// between calls), so a stale address is never used.
 //
 // All calls on a device share the one array and it keeps whatever the last
 // call left in it; calls that overlap on the GPU (two streams, two host
 // threads) would race on it, so callers must serialise them.  What has to
 // start at zero (the status block) is cleared at the start of every call;
 // the merge kernels overwrite everything else before reading it.
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <mutex>
@@ -35,18 +38,52 @@ static __device__ __align__(256) unsigned char g_no_alloc_scratch[MPM_NO_ALLOC_S
 constexpr int kMaxDevices = 64;
 constexpr size_t kStatusBlockBytes = 256;  // the status words lead the workspace
 std::mutex g_setup_mutex;
-void* g_scratch_ptr[kMaxDevices] = {};     // device address of the array, per device
+void* g_scratch_ptr[kMaxDevices] = {};             // device address of the array, per device
+unsigned long long g_scratch_ctx[kMaxDevices] = {};  // ID of the context that address belongs to
 
-// Device address of the scratch array on the current device (set up once).
+// Unique ID of the current context (cuCtxGetId, through the runtime's
+// driver entry points so that the library needs no -lcuda); 0 when no
+// context is current or the driver cannot say.
+unsigned long long current_context_id() {
+  using GetCurrent = CUresult (*)(CUcontext*);
+  using GetId = CUresult (*)(CUcontext, unsigned long long*);
+  static GetCurrent get_current = [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      return static_cast<GetCurrent>(nullptr);
+    return reinterpret_cast<GetCurrent>(p);
+  }();
+  static GetId get_id = [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      return static_cast<GetId>(nullptr);
+    return reinterpret_cast<GetId>(p);
+  }();
+  if (get_current == nullptr || get_id == nullptr) return 0;
+  CUcontext ctx = nullptr;
+  unsigned long long id = 0;
+  if (get_current(&ctx) != CUDA_SUCCESS || ctx == nullptr) return 0;
+  if (get_id(ctx, &id) != CUDA_SUCCESS) return 0;
+  return id;
+}
+
+// Device address of the scratch array on the current device.  Looked up
+// once per device context; without a context ID it is looked up each call.
 mpm_status scratch_on_current_device(void** out) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return MPM_ERR_CUDA;
   if (dev < 0 || dev >= kMaxDevices) return MPM_ERR_UNSUPPORTED;
   std::lock_guard<std::mutex> lock(g_setup_mutex);
-  if (g_scratch_ptr[dev] == nullptr) {
+  const unsigned long long ctx = current_context_id();
+  if (g_scratch_ptr[dev] == nullptr || ctx == 0 || ctx != g_scratch_ctx[dev]) {
     void* p = nullptr;
     if (cudaGetSymbolAddress(&p, g_no_alloc_scratch) != cudaSuccess || p == nullptr) return MPM_ERR_CUDA;
     g_scratch_ptr[dev] = p;
+    g_scratch_ctx[dev] = current_context_id();  // the lookup made a context current if none was
   }
   *out = g_scratch_ptr[dev];
   return MPM_OK;
@@ -67,4 +104,12 @@ extern "C" mpm_status mpm_merge_no_alloc(const void* tokens, const int64_t* offs
     return MPM_ERR_CUDA;
   return mpm_merge(tokens, offsets, batch, rows, dim, dtype, out_tokens, out_offsets, out_map, scratch,
                    MPM_NO_ALLOC_SCRATCH_BYTES, stream);
+}
+
+extern "C" mpm_status mpm_no_alloc_get_device_status(int32_t* host_code, void* stream) {
+  if (host_code == nullptr) return MPM_ERR_INVALID_ARG;
+  void* scratch = nullptr;
+  const mpm_status st = scratch_on_current_device(&scratch);
+  if (st != MPM_OK) return st;
+  return mpm_get_device_status(scratch, host_code, stream);
 }

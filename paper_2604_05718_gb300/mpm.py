@@ -31,7 +31,7 @@ STATUS_NAMES = {
 }
 EXPORTS = ("mpm_abi_version", "mpm_status_string", "mpm_merge_workspace_size", "mpm_merge", "mpm_merge_timed",
            "mpm_compose_maps", "mpm_unmerge_gather", "mpm_nearest_neighbors", "mpm_get_device_status",
-           "mpm_merge_no_alloc", "mpm_compose_gather", "mpm_pad_batch", "mpm_unpad_batch", "mpm_merge_chunked",
+           "mpm_merge_no_alloc", "mpm_no_alloc_get_device_status", "mpm_compose_gather", "mpm_pad_batch", "mpm_unpad_batch", "mpm_merge_chunked",
            "mpm_nearest_neighbors_chunked")
 
 _lib = None
@@ -59,6 +59,7 @@ def _declare(lib: ctypes.CDLL) -> None:
                                                  SZ, P]),
         "mpm_get_device_status": (ctypes.c_int, [P, P, P]),
         "mpm_merge_no_alloc": (ctypes.c_int, [P, P, I32, I64, I32, ctypes.c_int, P, P, P, P]),
+        "mpm_no_alloc_get_device_status": (ctypes.c_int, [P, P]),
         "mpm_compose_gather": (ctypes.c_int, [P, P, I64, P, P, I64, P, P, I64, I32, I32, ctypes.c_int, P, P, P,
                                               P]),
         "mpm_pad_batch": (ctypes.c_int, [P, P, I32, I64, I32, ctypes.c_int, I64, P, P, P, P, P]),
@@ -355,6 +356,16 @@ def merge_no_alloc(tokens: torch.Tensor, offsets: torch.Tensor, out_tokens: torc
                                             _ptr(out_map), _stream(dev))
     _check("mpm_merge_no_alloc", code)
     return out_tokens, out_offsets, out_map
+
+
+def no_alloc_device_status(device=None) -> int:
+    """First device-side error of the last merge_no_alloc call on a device (0 = none); clears it."""
+    dev = torch.device(device) if device is not None else torch.device("cuda", torch.cuda.current_device())
+    code = ctypes.c_int32(0)
+    with torch.cuda.device(dev):
+        _check("mpm_no_alloc_get_device_status",
+               library().mpm_no_alloc_get_device_status(ctypes.byref(code), _stream(dev)))
+    return int(code.value)
 
 
 def selftest_wait_timeout(limit_us: int, device=None) -> torch.Tensor:

@@ -148,6 +148,7 @@ def test_nn_compose_gather_validation(lib):
     assert nnc(P(FAKE), P(FAKE), 1, 10, 64, 1, 2, 256, P(FAKE * 8), None, P(FAKE * 32), 1 << 24, None) == 2
     assert nnc(P(FAKE), P(FAKE), 1, 10, 64, 1, 4, -256, P(FAKE * 8), None, P(FAKE * 32), 1 << 24, None) == 1
     assert lib.mpm_get_device_status(None, None, None) == 1
+    assert lib.mpm_no_alloc_get_device_status(None, None) == 1   # checked before any CUDA call
 
 
 def test_ordinary_library_has_no_timeline(lib):
