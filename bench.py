@@ -64,6 +64,8 @@ def parse_args():
     p.add_argument("--no-chunked", action="store_true", help="skip the chunked-similarity measurement")
     p.add_argument("--no-padded", action="store_true", help="skip the padded-batch measurement")
     p.add_argument("--no-fp32", action="store_true", help="skip the fp32 nearest-neighbour measurement")
+    p.add_argument("--no-per-workload", action="store_true",
+                   help="skip the step on the other four workloads (per_workload in the JSON line)")
     p.add_argument("--no-timeline", action="store_true",
                    help="skip the in-step device timeline (traced library, child process) of the default run")
     p.add_argument("--timeline", action="store_true",
@@ -88,20 +90,21 @@ def load_peaks():
         return dict(FALLBACK_PEAKS), "fallback"
 
 
-def workload_desc(cfg, batch):
+def workload_desc(cfg, batch, world=1):
     sizes = np.diff(batch.offsets)
     return {
         "workload": f"{cfg.name}: {cfg.description}",
-        "images": int(cfg.batch),
-        "tokens": int(batch.rows),
+        "images": int(world * cfg.batch),
+        "images_this_rank": int(batch.batch),
+        "tokens_this_rank": int(batch.rows),
         "tokens_per_image": int(sizes[0]) if len(set(sizes.tolist())) == 1 else "mixed",
         "dim": int(cfg.dim),
         "insertions": int(cfg.insertions),
         "seed": int(cfg.seed),
         "l2": "flushed before every step: 256 MiB written, then read back (clean lines)",
         "untimed": "the seeded N(0,0.05^2) stand-in for the encoder blocks between the two merges",
-        "parallelism": "image shards (rank r merges images r*B..(r+1)*B-1 of a world*B batch; "
-                       "no data-path collective)",
+        "parallelism": "image shards: each rank merges one contiguous range of the world*B images, "
+                       "balanced on sum(N_b^2) (shard.partition_images); no data-path collective",
     }
 
 
@@ -317,13 +320,238 @@ def traffic_for(kernel_files, rows_per_launch: float):
 # ---------------------------------------------------------------------------
 # The GPU path
 # ---------------------------------------------------------------------------
+# Nominal dense tf32 / bf16 tensor throughput (1.1 / 2.25 PFLOP/s per GB300):
+# the fp32 path's peak is the measured bf16 peak times this ratio.
+TF32_PER_BF16 = 1.1 / 2.25
+
+
+def new_events(stream, n):
+    """n timing events, recorded once so that their CUDA handles exist."""
+    import torch
+
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(n)]
+    for e in evs:
+        e.record(stream)
+    return evs
+
+
+class StepEvents:
+    """The CUDA events of one step."""
+
+    def __init__(self, stream):
+        self.seg = new_events(stream, 4)   # [merge1 start, merge1 end, rest start, rest end]
+        self.k1 = new_events(stream, 8)    # merge 1 kernels
+        self.k2 = new_events(stream, 8)    # merge 2 kernels
+        self.cg = new_events(stream, 2)    # around the (composed) gather
+
+
+class Step:
+    """Device buffers of one packed batch and the launches of one step.
+
+    merge (Algorithm 1) -> the untimed stand-in noise -> merge -> compose and
+    gather in one pass (Eq. 3 + Eq. 4); one insertion: merge -> gather.
+    """
+
+    def __init__(self, mpm, cfg, batch, images, dev, stream, flush, flush_sum):
+        import torch
+
+        from workloads import stage_noise
+
+        self.mpm, self.cfg, self.batch, self.stream = mpm, cfg, batch, stream
+        self.flush, self.flush_sum = flush, flush_sum
+        rows, dim, nimg = batch.rows, cfg.dim, batch.batch
+        self.x0 = batch.tokens.to(dev)
+        self.off0 = torch.from_numpy(batch.offsets).to(dev)
+        self.ws = mpm.new_workspace(rows, nimg, dim, self.x0.dtype, dev)
+        self.x1 = torch.empty_like(self.x0)
+        self.off1 = torch.empty(nimg + 1, dtype=torch.int64, device=dev)
+        self.m1 = torch.empty(rows, dtype=torch.int32, device=dev)
+        self.x1n = torch.zeros_like(self.x0)
+        self.x2 = torch.empty_like(self.x0)
+        self.off2 = torch.empty_like(self.off1)
+        self.m2 = torch.empty_like(self.m1)
+        self.rstar = torch.empty_like(self.m1)
+        self.up = torch.empty_like(self.x0)
+        self.two = cfg.insertions == 2
+        # One untimed pass fixes the stage-1 counts, hence the stand-in noise.
+        mpm.merge(self.x0, self.off0, workspace=self.ws, out_tokens=self.x1, out_offsets=self.off1,
+                  out_map=self.m1)
+        self.off1_h = self.off1.cpu().numpy()
+        self.t1 = int(self.off1_h[-1])
+        self.noise = (stage_noise(cfg.seed, np.diff(self.off1_h).tolist(), dim, images=images).to(dev)
+                      if self.two else None)
+
+    def launches(self) -> int:
+        """Kernels of the library launched by one step."""
+        return 2 * KERNELS_PER_MERGE + 1 if self.two else KERNELS_PER_MERGE + 1
+
+    def run(self, ev: StepEvents, host_in=None, host_out=None, per_kernel=False):
+        """One step; per_kernel adds CUDA events between the kernels (which
+        serialises them, so the step time is taken without them)."""
+        from workloads import apply_noise
+
+        mpm, s = self.mpm, self.stream
+        # Evict the L2: write 256 MiB, then read it back so that the lines left
+        # behind are clean (no write-back lands on the first timed kernel).
+        self.flush.fill_(1)
+        self.flush_sum.copy_(self.flush.view(self.flush_sum.dtype).sum())
+        ev.seg[0].record(s)
+        if host_in is not None:
+            self.x0.copy_(host_in[0], non_blocking=True)
+            self.off0.copy_(host_in[1], non_blocking=True)
+        mpm.merge(self.x0, self.off0, workspace=self.ws, out_tokens=self.x1, out_offsets=self.off1,
+                  out_map=self.m1, stage_events=ev.k1 if per_kernel else None)
+        ev.seg[1].record(s)
+        if self.two:
+            self.x1n[:self.t1] = apply_noise(self.x1[:self.t1], self.noise)
+        ev.seg[2].record(s)
+        if self.two:
+            mpm.merge(self.x1n, self.off1, workspace=self.ws, out_tokens=self.x2, out_offsets=self.off2,
+                      out_map=self.m2, stage_events=ev.k2 if per_kernel else None)
+            if per_kernel:
+                ev.cg[0].record(s)
+            # Eq. 3 and Eq. 4 in one pass; rstar receives the composed map.
+            mpm.compose_gather(self.x2, self.off2, self.m1, self.off0, self.m2, self.off1, out=self.up,
+                               out_map=self.rstar)
+        else:
+            if per_kernel:
+                ev.cg[0].record(s)
+            mpm.unmerge_gather(self.x1, self.off1, self.m1, self.off0, out=self.up)
+        if per_kernel:
+            ev.cg[1].record(s)
+        if host_out is not None:
+            host_out.copy_(self.up, non_blocking=True)
+        ev.seg[3].record(s)
+
+
+def time_step(p: Step, steps: int, warmup: int, barrier, max_over_ranks, clocks=None) -> dict:
+    """W warm-up steps, then K timed steps without and K with per-kernel events.
+
+    Returns the mean step time (max over ranks), the per-kernel means and
+    the affinity kernel's per-launch durations.
+    """
+    warm = StepEvents(p.stream)
+    for _ in range(warmup):
+        p.run(warm)
+    assert p.mpm.device_status(p.ws) == 0, "device status reported an error during warm-up"
+    events = [StepEvents(p.stream) for _ in range(steps)]
+    barrier()
+    if clocks is not None:
+        clocks.start()
+    wall0 = time.perf_counter()
+    for ev in events:
+        p.run(ev)
+    barrier()
+    wall = time.perf_counter() - wall0
+    clk = clocks.stop() if clocks is not None else None
+    seg_ms = [ev.seg[0].elapsed_time(ev.seg[1]) + ev.seg[2].elapsed_time(ev.seg[3]) for ev in events]
+    ms = max_over_ranks(statistics.mean(seg_ms))
+    assert p.mpm.device_status(p.ws) == 0, "device status reported an error in the timed loop"
+
+    # Second timed loop, same steps with CUDA events around every kernel: the
+    # per-kernel durations for the roofline and the breakdown.
+    kevents = [StepEvents(p.stream) for _ in range(steps)]
+    barrier()
+    for ev in kevents:
+        p.run(ev, per_kernel=True)
+    barrier()
+    ms_k = max_over_ranks(statistics.mean(
+        [ev.seg[0].elapsed_time(ev.seg[1]) + ev.seg[2].elapsed_time(ev.seg[3]) for ev in kevents]))
+
+    def kernel_ms(key, k):
+        return [getattr(ev, key)[2 * k].elapsed_time(getattr(ev, key)[2 * k + 1]) for ev in kevents]
+
+    kern = {}
+    for k, nm in enumerate(["prep", "affinity", "mutual_scan", "pair_average"]):
+        kern[f"{nm}_1_us"] = 1e3 * statistics.mean(kernel_ms("k1", k))
+        if p.two:
+            kern[f"{nm}_2_us"] = 1e3 * statistics.mean(kernel_ms("k2", k))
+    cg = [ev.cg[0].elapsed_time(ev.cg[1]) for ev in kevents]
+    kern["compose_gather_us" if p.two else "gather_us"] = 1e3 * statistics.mean(cg)
+    return {"ms": ms, "wall": wall, "clocks": clk, "ms_with_kernel_events": ms_k, "kern": kern,
+            "aff_ms_1": kernel_ms("k1", 1), "aff_ms_2": kernel_ms("k2", 1) if p.two else []}
+
+
+def step_metrics(p: Step, t: dict, peaks: dict, peak_kind: str) -> dict:
+    """Roofline figures of a timed step: the affinity kernel's algorithmic
+    flop rate and the bandwidth kernels' algorithmic byte rates."""
+    cfg, dim, kern = p.cfg, p.cfg.dim, t["kern"]
+    esize = 2 if cfg.dtype == "bf16" else 4
+    n0 = np.diff(p.batch.offsets).astype(np.float64)
+    n1 = np.diff(p.off1_h).astype(np.float64)
+    n2 = np.diff(p.off2.cpu().numpy()).astype(np.float64) if p.two else n1
+    # Algorithmic work of the affinity step: S is symmetric with a masked
+    # diagonal, so the minimum is the N(N-1)/2 off-diagonal dot products of
+    # D multiply-adds each, N(N-1)D flops per image per stage.
+    alg1 = float(np.sum(n0 * (n0 - 1.0) * dim))
+    alg2 = float(np.sum(n1 * (n1 - 1.0) * dim)) if p.two else 0.0
+    aff_ms = t["aff_ms_1"] + t["aff_ms_2"]
+    aff_flops = [alg1] * len(t["aff_ms_1"]) + [alg2] * len(t["aff_ms_2"])
+    achieved = sum(aff_flops) / (sum(aff_ms) * 1e-3) / 1e12
+    ratio = 1.0 if cfg.dtype == "bf16" else TF32_PER_BF16
+    burst = ratio * peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
+    sustained = ratio * peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
+    # What the tensor pipe executes (bf16): the 256 x 256 tiles on or above
+    # each image's diagonal, over K padded to 16 (the MMA's K).
+    kpad = -(-dim // 16) * 16
+
+    def exec_flops(ns):
+        r = -(-ns.astype(np.int64) // 256)
+        return float(np.sum(r * (r + 1) // 2)) * 256 * 256 * 2 * kpad
+
+    exe = [exec_flops(n0)] * len(t["aff_ms_1"]) + [exec_flops(n1)] * len(t["aff_ms_2"])
+    executed = sum(exe) / (sum(aff_ms) * 1e-3) / 1e12 if cfg.dtype == "bf16" else None
+    hbm = peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
+
+    def gbs(nbytes, us):
+        return nbytes / (us * 1e-6) / 1e9
+
+    bw = {
+        "prep_1_gbs": gbs(n0.sum() * dim * esize + 12 * n0.sum(), kern["prep_1_us"]),
+        "pair_average_1_gbs": gbs((n0.sum() + n1.sum()) * dim * esize + 12 * n0.sum(), kern["pair_average_1_us"]),
+    }
+    if p.two:
+        bw["prep_2_gbs"] = gbs(n1.sum() * dim * esize + 12 * n1.sum(), kern["prep_2_us"])
+        bw["pair_average_2_gbs"] = gbs((n1.sum() + n2.sum()) * dim * esize + 12 * n1.sum(),
+                                       kern["pair_average_2_us"])
+    # Gather reads each merged row it needs and writes the grid; with two
+    # insertions it also reads both maps and writes the composed one.
+    bw["gather_gbs"] = gbs((n2.sum() + n0.sum()) * dim * esize + (12 if p.two else 4) * n0.sum(),
+                           kern["compose_gather_us" if p.two else "gather_us"])
+    for k in list(bw):
+        bw[k.replace("_gbs", "_frac")] = bw[k] / hbm
+    return {"n0": n0, "n1": n1, "n2": n2, "alg1": alg1, "alg2": alg2,
+            "aff_launches": len(aff_ms), "aff_flops_per_launch": sum(aff_flops) / len(aff_ms),
+            "aff_tflops": achieved, "aff_peak_burst": burst, "aff_peak_sustained": sustained,
+            "aff_executed_tflops": executed, "hbm": bw, "hbm_peak": hbm,
+            "rows_per_aff_launch": (n0.sum() + (n1.sum() if p.two else 0.0)) / (2.0 if p.two else 1.0)}
+
+
+def workload_summary(p: Step, t: dict, m: dict) -> dict:
+    """The per-workload record of the JSON line."""
+    out = {
+        "images": p.batch.batch, "tokens": p.batch.rows, "dim": p.cfg.dim, "dtype": p.cfg.dtype,
+        "insertions": p.cfg.insertions, "ms_per_step": t["ms"],
+        "images_per_s": p.batch.batch / (t["ms"] * 1e-3), "tokens_per_s": p.batch.rows / (t["ms"] * 1e-3),
+        "affinity_tflops_algorithmic": m["aff_tflops"],
+        "affinity_frac_of_burst": m["aff_tflops"] / m["aff_peak_burst"],
+        "affinity_frac_of_sustained": m["aff_tflops"] / m["aff_peak_sustained"],
+        "affinity_peak": ("bf16 dense" if p.cfg.dtype == "bf16" else
+                          "tf32 dense = bf16 x 1.1/2.25 (nominal ratio); three tf32 products per term"),
+        "affinity_us": {k: v for k, v in t["kern"].items() if k.startswith("affinity")},
+    }
+    out.update({k: v for k, v in m["hbm"].items() if k.endswith("_frac")})
+    return out
+
+
 def run_mpm(args):
     import torch
     import torch.distributed as dist
 
     import paper_2604_05718_gb300 as mpm
     from paper_2604_05718_gb300 import build
-    from workloads import CONFIGS, WorkloadConfig, apply_noise, make_batch, stage_noise
+    from paper_2604_05718_gb300.shard import partition_images
+    from workloads import CONFIG_ORDER, CONFIGS, WorkloadConfig, apply_noise, image_shape, make_batch
 
     rank, world, local = dist_env()
     if not torch.cuda.is_available():
@@ -336,10 +564,17 @@ def run_mpm(args):
     mpm.library()
 
     cfg = CONFIGS[args.workload]
-    # Rank r merges images [r*B, (r+1)*B) of a global batch of world*B images.
-    images = list(range(rank * cfg.batch, (rank + 1) * cfg.batch))
+    # The global batch holds world x B images of the workload.  Rank r merges
+    # one contiguous range of them, balanced on sum(N_b^2) (the affinity
+    # cost); images are independent, so no data crosses ranks.
+    global_images = world * cfg.batch
+    sizes = [image_shape(cfg, b)[0] ** 2 for b in range(global_images)]
+    lo, hi = partition_images(sizes, world)[rank]
+    if hi <= lo:
+        raise RuntimeError(f"rank {rank} received no images of the {global_images}-image batch")
+    images = list(range(lo, hi))
     batch = make_batch(cfg, images=images)
-    rows, dim, nimg = batch.rows, cfg.dim, cfg.batch
+    rows, dim, nimg = batch.rows, cfg.dim, batch.batch
     esize = 2 if cfg.dtype == "bf16" else 4
     stream = torch.cuda.current_stream(dev)
 
@@ -349,74 +584,12 @@ def run_mpm(args):
         n_img, secs = oracle_sample(cfg, batch, args.cpu_seconds)
         cpu_base = cpu_baseline_obj(n_img, secs, cfg)
 
-    x0 = batch.tokens.to(dev)
-    off0 = torch.from_numpy(batch.offsets).to(dev)
-    ws = mpm.new_workspace(rows, nimg, dim, x0.dtype, dev)
-    x1 = torch.empty_like(x0)
-    off1 = torch.empty(nimg + 1, dtype=torch.int64, device=dev)
-    m1 = torch.empty(rows, dtype=torch.int32, device=dev)
-    x1n = torch.zeros_like(x0)
-    x2 = torch.empty_like(x0)
-    off2 = torch.empty_like(off1)
-    m2 = torch.empty_like(m1)
-    rstar = torch.empty_like(m1)
-    up = torch.empty_like(x0)
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     flush_sum = torch.zeros((), dtype=torch.int64, device=dev)
-
-    # One untimed pass fixes the stage-1 counts, hence the stand-in noise.
-    mpm.merge(x0, off0, workspace=ws, out_tokens=x1, out_offsets=off1, out_map=m1)
-    off1_h = off1.cpu().numpy()
-    t1 = int(off1_h[-1])
-    two = cfg.insertions == 2
-    noise = stage_noise(cfg.seed, np.diff(off1_h).tolist(), dim, images=images).to(dev) if two else None
-
-    def new_events(n):
-        evs = [torch.cuda.Event(enable_timing=True) for _ in range(n)]
-        for e in evs:
-            e.record(stream)  # materialise the CUDA event handles
-        return evs
-
-    class StepEvents:
-        def __init__(self):
-            self.seg = new_events(4)       # [merge1 start, merge1 end, rest start, rest end]
-            self.k1 = new_events(8)        # merge 1 kernels
-            self.k2 = new_events(8)        # merge 2 kernels
-            self.cg = new_events(2)        # around the (composed) gather
-
-    def step(ev: StepEvents, host_in=None, host_out=None, per_kernel=False):
-        """One step; per_kernel adds CUDA events between the kernels (which
-        serialises them, so the step time is taken without them)."""
-        # Evict the L2: write 256 MiB, then read it back so that the lines left
-        # behind are clean (no write-back lands on the first timed kernel).
-        flush.fill_(1)
-        flush_sum.copy_(flush.view(torch.int64).sum())
-        ev.seg[0].record(stream)
-        if host_in is not None:
-            x0.copy_(host_in[0], non_blocking=True)
-            off0.copy_(host_in[1], non_blocking=True)
-        mpm.merge(x0, off0, workspace=ws, out_tokens=x1, out_offsets=off1, out_map=m1,
-                  stage_events=ev.k1 if per_kernel else None)
-        ev.seg[1].record(stream)
-        if two:
-            x1n[:t1] = apply_noise(x1[:t1], noise)
-        ev.seg[2].record(stream)
-        if two:
-            mpm.merge(x1n, off1, workspace=ws, out_tokens=x2, out_offsets=off2, out_map=m2,
-                      stage_events=ev.k2 if per_kernel else None)
-            if per_kernel:
-                ev.cg[0].record(stream)
-            # Eq. 3 and Eq. 4 in one pass; rstar receives the composed map.
-            mpm.compose_gather(x2, off2, m1, off0, m2, off1, out=up, out_map=rstar)
-        else:
-            if per_kernel:
-                ev.cg[0].record(stream)
-            mpm.unmerge_gather(x1, off1, m1, off0, out=up)
-        if per_kernel:
-            ev.cg[1].record(stream)
-        if host_out is not None:
-            host_out.copy_(up, non_blocking=True)
-        ev.seg[3].record(stream)
+    p = Step(mpm, cfg, batch, images, dev, stream, flush, flush_sum)
+    x0, off0, ws, x1, off1, m1 = p.x0, p.off0, p.ws, p.x1, p.off1, p.m1
+    x1n, x2, off2, m2, rstar, up = p.x1n, p.x2, p.off2, p.m2, p.rstar, p.up
+    t1, two, noise = p.t1, p.two, p.noise
 
     def barrier():
         torch.cuda.synchronize(dev)
@@ -432,103 +605,46 @@ def run_mpm(args):
         return float(t.item())
 
     # ---------------- device-resident timed loop ----------------
-    events = [StepEvents() for _ in range(args.steps)]
-    warm = StepEvents()
-    for _ in range(args.warmup):
-        step(warm)
-    assert mpm.device_status(ws) == 0, "device status reported an error during warm-up"
-    clocks = ClockSampler(dev)
-    barrier()
-    clocks.start()
-    wall0 = time.perf_counter()
-    for ev in events:
-        step(ev)
-    barrier()
-    wall = time.perf_counter() - wall0
-    clk = clocks.stop()
-    seg_ms = [ev.seg[0].elapsed_time(ev.seg[1]) + ev.seg[2].elapsed_time(ev.seg[3]) for ev in events]
-    ms = max_over_ranks(statistics.mean(seg_ms))
-    off2_h = off2.cpu().numpy() if two else off1_h
-    assert mpm.device_status(ws) == 0, "device status reported an error in the timed loop"
-
-    # Second timed loop, same steps with CUDA events around every kernel: the
-    # per-kernel durations for the roofline and the breakdown.
-    kevents = [StepEvents() for _ in range(args.steps)]
-    barrier()
-    for ev in kevents:
-        step(ev, per_kernel=True)
-    barrier()
-    ms_with_kernel_events = max_over_ranks(statistics.mean(
-        [ev.seg[0].elapsed_time(ev.seg[1]) + ev.seg[2].elapsed_time(ev.seg[3]) for ev in kevents]))
-
-    # Per-kernel durations inside the timed region.
-    def kernel_ms(key, k):
-        return [getattr(ev, key)[2 * k].elapsed_time(getattr(ev, key)[2 * k + 1]) for ev in kevents]
-
-    names = ["prep", "affinity", "mutual_scan", "pair_average"]
-    kern = {}
-    for k, nm in enumerate(names):
-        kern[f"{nm}_1_us"] = 1e3 * statistics.mean(kernel_ms("k1", k))
-        if two:
-            kern[f"{nm}_2_us"] = 1e3 * statistics.mean(kernel_ms("k2", k))
-    cg = [ev.cg[0].elapsed_time(ev.cg[1]) for ev in kevents]
-    kern["gather_us" if not two else "compose_gather_us"] = 1e3 * statistics.mean(cg)
-
+    t = time_step(p, args.steps, args.warmup, barrier, max_over_ranks, ClockSampler(dev))
+    ms, wall, clk, kern = t["ms"], t["wall"], t["clocks"], t["kern"]
+    ms_with_kernel_events = t["ms_with_kernel_events"]
     peaks, peak_kind = load_peaks()
-    n0 = np.diff(batch.offsets).astype(np.float64)
-    n1 = np.diff(off1_h).astype(np.float64)
-    n2 = np.diff(off2_h).astype(np.float64)
-    # Algorithmic work of the affinity step: S is symmetric with a masked
-    # diagonal, so the minimum is the N(N-1)/2 off-diagonal dot products of
-    # D multiply-adds each, N(N-1)D flops per image per stage.
-    alg1 = float(np.sum(n0 * (n0 - 1.0) * dim))
-    alg2 = float(np.sum(n1 * (n1 - 1.0) * dim)) if two else 0.0
-    aff_ms = kernel_ms("k1", 1) + (kernel_ms("k2", 1) if two else [])
-    aff_flops = [alg1] * args.steps + ([alg2] * args.steps if two else [])
-    launches = len(aff_ms)
-    achieved_tflops = sum(aff_flops) / (sum(aff_ms) * 1e-3) / 1e12
-    flops_per_launch = sum(aff_flops) / launches
-    tensor_peak = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
-    # What the tensor pipe executes: the 256 x 256 tiles on or above each
-    # image's diagonal, over K padded to 16 (the MMA's K).
-    kpad = -(-dim // 16) * 16
-
-    def exec_flops(ns):
-        r = -(-ns.astype(np.int64) // 256)
-        return float(np.sum(r * (r + 1) // 2)) * 256 * 256 * 2 * kpad
-
-    exe = [exec_flops(n0)] * args.steps + ([exec_flops(n1)] * args.steps if two else [])
-    executed_tflops = sum(exe) / (sum(aff_ms) * 1e-3) / 1e12
-    rows_per_launch = (n0.sum() + (n1.sum() if two else 0.0)) / (2.0 if two else 1.0)
-    traffic = traffic_for(AFFINITY_SOURCES, rows_per_launch)
+    m = step_metrics(p, t, peaks, peak_kind)
+    n0, n1, n2 = m["n0"], m["n1"], m["n2"]
     roofline = {
         "kernel": "affinity_pair_kernel (fused cosine affinity + arg max, TMA + tcgen05.mma.cta_group::2)",
-        "bound": "tensor", "achieved": achieved_tflops, "peak": tensor_peak, "unit": "TFLOP/s",
-        "frac": achieved_tflops / tensor_peak,
-        "peak_kind": f"{peak_kind} bf16 sustained (kernel timed inside the step loop)",
-        "flops_per_launch": flops_per_launch,
+        "bound": "tensor", "achieved": m["aff_tflops"], "peak": m["aff_peak_burst"], "unit": "TFLOP/s",
+        "frac": m["aff_tflops"] / m["aff_peak_burst"],
+        "peak_kind": (f"{peak_kind} bf16 burst: the timed region is {args.steps} steps of well under a "
+                      "millisecond each, not a seconds-long loop"),
+        "peak_sustained": m["aff_peak_sustained"],
+        "frac_of_sustained": m["aff_tflops"] / m["aff_peak_sustained"],
+        "flops_per_launch": m["aff_flops_per_launch"],
         "flops_definition": "algorithmic: N_b (N_b - 1) D per image per stage (off-diagonal half of S = X X^T)",
-        "frac_of_burst_peak": achieved_tflops / peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]),
-        "executed_tflops": executed_tflops,
-        "executed_frac": executed_tflops / tensor_peak,
+        "executed_tflops": m["aff_executed_tflops"],
+        "executed_frac": (m["aff_executed_tflops"] / m["aff_peak_burst"]
+                          if m["aff_executed_tflops"] is not None else None),
         "executed_definition": "MMA work issued: 256x256 tiles on or above the diagonal x K padded to 16",
-        "traffic": traffic,
+        "traffic": traffic_for(AFFINITY_SOURCES, m["rows_per_aff_launch"]),
     }
-    # HBM fractions of the bandwidth kernels (algorithmic bytes / event time).
-    hbm = peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
-    avg1 = float((n0.sum() + n1.sum()) * dim * esize + 12 * n0.sum())
-    # Gather reads each merged row it needs and writes the grid; with two
-    # insertions it also reads both maps and writes the composed one.
-    gat = float((n2.sum() + n0.sum()) * dim * esize + (12 if two else 4) * n0.sum())
-    norm1 = float(n0.sum() * dim * esize + 12 * n0.sum())
-    hbm_kernels = {
-        "pair_average_1_gbs": avg1 / (kern["pair_average_1_us"] * 1e-6) / 1e9,
-        "gather_gbs": gat / (kern["gather_us" if not two else "compose_gather_us"] * 1e-6) / 1e9,
-        "prep_1_gbs": norm1 / (kern["prep_1_us"] * 1e-6) / 1e9,
-        "peak_gbs": hbm, "peak_kind": f"{peak_kind} copy bandwidth",
-    }
-    for k in ("pair_average_1", "gather", "prep_1"):
-        hbm_kernels[k + "_frac"] = hbm_kernels[k + "_gbs"] / hbm
+    hbm_kernels = dict(m["hbm"], peak_gbs=m["hbm_peak"], peak_kind=f"{peak_kind} copy bandwidth")
+
+    # ---------------- every workload, the same step (one GPU) ----------------
+    per_workload = None
+    if world == 1 and not args.no_per_workload:
+        per_workload = {}
+        pw_steps, pw_warm = min(args.steps, 50), max(3, min(args.warmup, 5))
+        for name in CONFIG_ORDER:
+            if name == args.workload:
+                per_workload[name] = dict(workload_summary(p, t, m), steps=args.steps)
+                continue
+            wcfg = CONFIGS[name]
+            wb = make_batch(wcfg)
+            wp = Step(mpm, wcfg, wb, list(range(wcfg.batch)), dev, stream, flush, flush_sum)
+            wt = time_step(wp, pw_steps, pw_warm, barrier, max_over_ranks)
+            per_workload[name] = dict(workload_summary(wp, wt, step_metrics(wp, wt, peaks, peak_kind)),
+                                      steps=pw_steps)
+            del wp, wb
 
     # ---------------- padded batch of the stage-1 output (next-step consumer layout) ----------------
     # The merged sequences padded to the longest one, with a key mask, as the
@@ -543,7 +659,7 @@ def run_mpm(args):
     for it in range(0 if args.no_padded else max(3, args.warmup) + 20):
         flush.fill_(1)
         flush_sum.copy_(flush.view(torch.int64).sum())
-        e = new_events(3)
+        e = new_events(stream, 3)
         e[0].record(stream)
         mpm.pad_batch(x1, off1, n1_max, out=pad_out, mask=pad_mask, stats=pad_stats)
         e[1].record(stream)
@@ -586,7 +702,7 @@ def run_mpm(args):
             for it in range(max(3, args.warmup) + 20):
                 flush.fill_(1)
                 flush_sum.copy_(flush.view(torch.int64).sum())
-                e = new_events(2)
+                e = new_events(stream, 2)
                 e[0].record(stream)
                 mpm.merge(mx, moff, workspace=mws, out_tokens=mout, out_offsets=moo, out_map=mmap, chunk=chunk)
                 e[1].record(stream)
@@ -618,7 +734,7 @@ def run_mpm(args):
             for it in range(max(3, args.warmup) + 10):
                 flush.fill_(1)
                 flush_sum.copy_(flush.view(torch.int64).sum())
-                e = new_events(2)
+                e = new_events(stream, 2)
                 e[0].record(stream)
                 nn_f, _ = mpm.nearest_neighbors(fx, foff, algo=algo, workspace=fws, with_score=False)
                 e[1].record(stream)
@@ -698,7 +814,7 @@ def run_mpm(args):
         # The copied-back grids must be the device result.
         for sl in range(2):
             assert torch.equal(host_up[sl].to(dev), up), "copied-back grid differs from the device result"
-        e2e = {"value": world * nimg / (e_ms * 1e-3), "unit": UNIT,
+        e2e = {"value": global_images / (e_ms * 1e-3), "unit": UNIT,
                "h2d_bytes_per_step": int(host_x.numel() * host_x.element_size() + host_off.numel() * 8),
                "d2h_bytes_per_step": int(host_up[0].numel() * host_up[0].element_size()),
                "ms_per_step": e_ms,
@@ -716,14 +832,15 @@ def run_mpm(args):
         dist.barrier()
     if rank == 0:
         line = {
-            "metric": METRIC, "value": world * nimg / (ms * 1e-3), "unit": UNIT, "n_gpus": world,
+            "metric": METRIC, "value": global_images / (ms * 1e-3), "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": cfg.dtype, "data": "synthetic",
-            "config": workload_desc(cfg, batch),
-            "tokens_per_s": world * rows / (ms * 1e-3),
+            "config": workload_desc(cfg, batch, world),
+            "tokens_per_s": float(sum(sizes)) / (ms * 1e-3),
             "merged_tokens": {"stage0": int(n0.sum()), "stage1": int(n1.sum()), "stage2": int(n2.sum())},
             "roofline": roofline,
             "hbm_kernels": hbm_kernels,
+            "per_workload": per_workload,
             "padded_batch": padded,
             "chunked_similarity": chunked,
             "fp32_nearest_neighbours": fp32,
@@ -733,7 +850,7 @@ def run_mpm(args):
             "cpu_baseline": cpu_base,
             "e2e": e2e,
             "clocks": clk,
-            "gpu_launches": (2 * KERNELS_PER_MERGE + 1 if two else KERNELS_PER_MERGE + 1) * args.steps,
+            "gpu_launches": p.launches() * args.steps,
             "wall_s_timed_loop": wall,
         }
         print(json.dumps(line), flush=True)

@@ -38,6 +38,14 @@ def test_gpu_arm_prints_one_contract_line():
     c = d["clocks"]
     assert {"sm_mhz", "sm_max_mhz", "reasons"} <= set(c)
     assert d["gpu_launches"] == 9 * d["steps"]   # four kernels per merge, two merges, one compose + gather
+    # Every workload's step, measured in the same run.
+    pw = d["per_workload"]
+    assert set(pw) == {"vit_t_single", "vit_s", "vit_b", "vit_l", "mixed"}
+    for name, w in pw.items():
+        assert w["images_per_s"] > 0 and w["tokens_per_s"] > 0, name
+        assert 0 < w["affinity_frac_of_burst"] < 1.5 and 0 < w["gather_frac"] < 1.5, name
+        assert 0 < w["pair_average_1_frac"] < 1.5 and 0 < w["prep_1_frac"] < 1.5, name
+    assert abs(pw["vit_b"]["images_per_s"] - d["value"]) < 1e-6 * d["value"]
     # The in-step timeline of the traced library, beside the event figures.
     ins = d["in_step"]
     assert ins is not None and ins["affinity_tflops_algorithmic"] > 0
