@@ -27,6 +27,13 @@
 //    i by G_ij / |x_i|), as in affinity_tc.cu's symmetric mode; the block
 //    below the diagonal of a diagonal tile is skipped.
 //
+// Rows of the tile are assigned crosswise: the leader CTA (rank 0, whose
+// warp 1 issues the MMAs) holds tile rows [128, 256) and the peer rows
+// [0, 128).  In a diagonal tile the rows [128, 256) skip the block below the
+// diagonal, so the lighter half of the epilogue runs on the SM that also
+// issues the MMAs: epilogue instructions on the issuing warp's SM
+// sub-partition are what slows the MMA issue.
+//
 // Roles per CTA (10 warps): warp 0 loads its CTA's A and B slices with TMA
 // and reports the bytes to the leader CTA's barrier; in the leader, warp 1
 // allocates tensor memory (jointly with the peer) and issues the MMAs, whose
@@ -365,7 +372,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       bool ok = true;
       for (int64_t k = 0; ok && k < count; ++k) {
         const Item it = item(k);
-        const int32_t arow = static_cast<int32_t>(it.base + it.row0 + HALF * rank);
+        const int32_t arow = static_cast<int32_t>(it.base + it.row0 + HALF * (rank ^ 1u));
         const int32_t brow = static_cast<int32_t>(it.base + it.col0 + HALF * rank);
         for (int kb = 0; kb < ksteps; ++kb) {
           if (!ptx::mbar_wait(&ctl->empty[stage], phase ^ 1u, abort_flag, WAIT_LIMIT_NS)) {
@@ -490,8 +497,8 @@ __global__ void __launch_bounds__(THREADS, 1)
         const int j = nx.col0 + c0 + 32 * h + lane;
         pf_scale[h] = j < nx.n ? __ldg(ws.inv_norm + nx.base + j) : nan;
       }
-      const int r = nx.row0 + HALF * static_cast<int>(rank) + q * 32 + lane;
-      const bool col = (nx.col0 + c0) / HALF > (nx.row0 + HALF * static_cast<int>(rank)) / HALF;
+      const int r = nx.row0 + HALF * static_cast<int>(rank ^ 1u) + q * 32 + lane;
+      const bool col = (nx.col0 + c0) / HALF > (nx.row0 + HALF * static_cast<int>(rank ^ 1u)) / HALF;
       pf_inv = (col && r < nx.n) ? __ldg(ws.inv_norm + nx.base + r) : 0.f;
     };
     const uint32_t empty_leader0 = map_to_rank(ptx::smem_addr(&ctl->acc_empty[0]), 0);
@@ -509,10 +516,10 @@ __global__ void __launch_bounds__(THREADS, 1)
       }
       if (k + 1 < count) prefetch(item(k + 1));
       ptx::tc_fence_after_sync();
-      const int row_base = it.row0 + HALF * static_cast<int>(rank) + q * 32;
+      const int row_base = it.row0 + HALF * static_cast<int>(rank ^ 1u) + q * 32;
       const int row = row_base + lane;
       const int jd = row - it.col0;
-      const int iblk = (it.row0 + HALF * static_cast<int>(rank)) / HALF;
+      const int iblk = (it.row0 + HALF * static_cast<int>(rank ^ 1u)) / HALF;
       const int jblk = (it.col0 + c0) / HALF;
       const bool diag = jblk == iblk;
       const bool col_update = jblk > iblk;
