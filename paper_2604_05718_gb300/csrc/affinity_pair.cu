@@ -34,12 +34,13 @@
 // issues the MMAs: epilogue instructions on the issuing warp's SM
 // sub-partition are what slows the MMA issue.
 //
-// Roles per CTA (10 warps): warp 0 loads its CTA's A and B slices with TMA
-// and reports the bytes to the leader CTA's barrier; in the leader, warp 1
+// Roles per CTA (2 + EPIW warps): warp 0 loads its CTA's A and B slices with
+// TMA and reports the bytes to the leader CTA's barrier; in the leader, warp 1
 // allocates tensor memory (jointly with the peer) and issues the MMAs, whose
-// completion is multicast to both CTAs; warps 2-9 of each CTA read their own
-// tensor memory in 32 x 128 slices.  Every wait is bounded; on expiry the
-// kernel records MPM_ERR_DEVICE_TIMEOUT and unwinds.
+// completion is multicast to both CTAs; the other warps of each CTA read
+// their own tensor memory in slices of 32 rows x 128 columns (EPIW = 8) or
+// 32 x 64 (EPIW = 16, rows of few features).  Every wait is bounded; on
+// expiry the kernel records MPM_ERR_DEVICE_TIMEOUT and unwinds.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <math.h>
@@ -63,13 +64,21 @@ constexpr int ATOM_BYTES = HALF * BOX_K * 2;   // 16 KiB
 constexpr int STAGES = 3;
 constexpr int SLICE_BYTES = ATOMS * ATOM_BYTES;  // 32 KiB: 128 rows x BK features
 constexpr int STAGE_BYTES = 2 * SLICE_BYTES;     // A slice + B slice of this CTA
-// Epilogue warps: two per SM sub-partition, each reading 32 TMEM lanes x 128
-// columns.  Fewer, longer epilogue warps leave the MMA-issuing warp more of
-// its sub-partition's issue slots (measured: 8 warps beat 16 and 4).
-constexpr int EPI_WARPS = 8;
-constexpr int EPI_COLS = TILE / (EPI_WARPS / 4);
-static_assert(EPI_COLS <= HALF && HALF % EPI_COLS == 0, "a warp's columns lie in one 128-column block");
-constexpr int THREADS = (2 + EPI_WARPS) * 32;
+// Epilogue warps: EPIW per CTA, EPIW / 4 per SM sub-partition, each reading
+// 32 TMEM lanes x TILE / (EPIW / 4) columns.  Eight (two per sub-partition,
+// 128 columns each) leave the MMA-issuing warp most of its sub-partition's
+// issue slots, which bounds tiles of many features (measured: 8 warps beat
+// 16 and 4 at D = 768 and 1024).  With few features a tile's MMAs are short
+// and its epilogue, latency-bound, sets the pace; sixteen warps of 64
+// columns hide more of that latency (D = 384: 26.6 instead of 28.6 us).
+template <int EPIW>
+struct Epi {
+  static constexpr int WARPS = EPIW;
+  static constexpr int COLS = TILE / (EPIW / 4);
+  static constexpr int THREADS = (2 + EPIW) * 32;
+  static_assert(COLS <= HALF && HALF % COLS == 0 && COLS % 32 == 0, "a warp's columns lie in one 128-column block");
+};
+constexpr int kWideEpilogueMaxDim = 512;  // bf16 rows of at most this many features take 16 epilogue warps
 constexpr uint32_t TMEM_COLS = 2 * TILE;
 constexpr uint32_t IDESC = ptx::idesc_bf16_f32(2 * HALF, TILE);
 // fp32 tokens: three tf32 products per K slice (hi hi + hi lo + lo hi, the
@@ -101,9 +110,12 @@ struct Item {
   int origin;    // index of the chunk's first token within its image
 };
 
-constexpr size_t SMEM_BYTES = 1024 + static_cast<size_t>(STAGES) * STAGE_BYTES + EPI_WARPS * EPI_COLS * sizeof(float) +
-                              sizeof(Control) + 16 + kMaxItems * sizeof(Item) +
-                              2 * (kMaxStagedImages + 1) * sizeof(int64_t) + EPI_WARPS * 32 * sizeof(uint2);
+template <int EPIW>
+constexpr size_t smem_bytes() {
+  return 1024 + static_cast<size_t>(STAGES) * STAGE_BYTES + Epi<EPIW>::WARPS * Epi<EPIW>::COLS * sizeof(float) +
+         sizeof(Control) + 16 + kMaxItems * sizeof(Item) + 2 * (kMaxStagedImages + 1) * sizeof(int64_t) +
+         Epi<EPIW>::WARPS * 32 * sizeof(uint2);
+}
 
 // Item w of the launch: image by the plan, its chunk, then the
 // upper-triangle tile (I, J), J >= I, of that chunk numbered row by row: row
@@ -286,11 +298,14 @@ __device__ __forceinline__ void fail(Control* ctl, int32_t* status, int32_t role
 
 // TF32: fp32 tokens through the three-product tf32 split (tmap = high
 // parts, tmap_lo = low parts); otherwise bf16 tokens (tmap_lo unused).
-template <bool TF32>
-__global__ void __launch_bounds__(THREADS, 1)
+template <bool TF32, int EPIW>
+__global__ void __launch_bounds__(Epi<EPIW>::THREADS, 1)
     affinity_pair_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constant__ CUtensorMap tmap_lo,
                          int batch, int dim, int64_t chunk, Workspace ws) {
   constexpr int kBK = TF32 ? TF_BK : BK;
+  constexpr int EPI_WARPS = Epi<EPIW>::WARPS;
+  constexpr int EPI_COLS = Epi<EPIW>::COLS;
+  constexpr int THREADS = Epi<EPIW>::THREADS;
   MPM_TRACE_BEGIN(MPM_TRACE_AFFINITY);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024u - (ptx::smem_addr(smem_raw) & 1023u)) & 1023u);
@@ -608,22 +623,29 @@ cudaError_t launch_affinity_pair(const void* tokens, int batch, int64_t rows, in
              CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) !=
           CUDA_SUCCESS)
     return cudaErrorInvalidValue;
-  static std::atomic<uint64_t> attr_done[2] = {{0}, {0}};
+  // Kernel instances: fp32 tokens (8 epilogue warps), bf16 with 8, bf16 with
+  // 16 (rows of at most kWideEpilogueMaxDim features).
+  static std::atomic<uint64_t> attr_done[3] = {{0}, {0}, {0}};
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   const uint64_t bit = 1ull << (dev & 63);
-  auto kernel = tf32 ? affinity_pair_kernel<true> : affinity_pair_kernel<false>;
-  if (!(attr_done[tf32].load() & bit)) {
-    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(SMEM_BYTES));
+  const int inst = tf32 ? 0 : (dim <= kWideEpilogueMaxDim ? 2 : 1);
+  void (*const kernels[3])(CUtensorMap, CUtensorMap, int, int, int64_t, Workspace) = {
+      affinity_pair_kernel<true, 8>, affinity_pair_kernel<false, 8>, affinity_pair_kernel<false, 16>};
+  const size_t smem[3] = {smem_bytes<8>(), smem_bytes<8>(), smem_bytes<16>()};
+  const int threads[3] = {Epi<8>::THREADS, Epi<8>::THREADS, Epi<16>::THREADS};
+  auto kernel = kernels[inst];
+  if (!(attr_done[inst].load() & bit)) {
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem[inst]));
     if (e != cudaSuccess) return e;
-    attr_done[tf32].fetch_or(bit);
+    attr_done[inst].fetch_or(bit);
   }
   const int grid = (num_sms > 1 ? num_sms : 2) & ~1;  // whole SM pairs
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
-  cfg.blockDim = dim3(THREADS);
-  cfg.dynamicSmemBytes = SMEM_BYTES;
+  cfg.blockDim = dim3(threads[inst]);
+  cfg.dynamicSmemBytes = smem[inst];
   cfg.stream = stream;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
