@@ -194,8 +194,10 @@ def test_merge_is_bitwise_deterministic(mpm, dtype):
                            other[0].view(torch.int16 if dtype == "bf16" else torch.int32))
 
 
-def test_tcgen05_and_simt_agree(mpm):
-    batch = make_custom([1000, 513, 64, 2300], 384, "bf16", seed=9)
+@pytest.mark.parametrize("dim", [384, 768])
+def test_tcgen05_and_simt_agree(mpm, dim):
+    # D = 384 runs the SM-pair kernel with 16 epilogue warps, D = 768 with 8.
+    batch = make_custom([1000, 513, 64, 2300], dim, "bf16", seed=9)
     runs = {algo: run_merge(mpm, batch.tokens, batch.offsets, algo)
             for algo in ("tcgen05", "tcgen05_sym", "tcgen05_pair", "simt")}
     res = [oracle.merge_image(batch.tokens[batch.offsets[k]:batch.offsets[k + 1]].double().numpy())
