@@ -43,9 +43,11 @@ def run(mpm, batch, chunk, algo="auto"):
     return nn.cpu().numpy(), rmap.cpu().numpy(), to_f64(out[:t]), out_off.cpu().numpy()
 
 
+@pytest.mark.parametrize("dim", [128, 768])
 @pytest.mark.parametrize("chunk", [256, 512])
-def test_chunked_bf16_matches_oracle(mpm, chunk):
-    batch = make_custom(COUNTS, 128, "bf16", seed=41)
+def test_chunked_bf16_matches_oracle(mpm, chunk, dim):
+    # D = 128 runs the SM-pair kernel with 16 epilogue warps, D = 768 with 8.
+    batch = make_custom(COUNTS, dim, "bf16", seed=41)
     nn, rmap, out, out_off = run(mpm, batch, chunk)
     # No neighbour crosses a chunk; a token alone in its chunk has none.
     for b in range(batch.batch):
