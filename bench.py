@@ -506,24 +506,42 @@ def step_metrics(p: Step, t: dict, peaks: dict, peak_kind: str) -> dict:
     def gbs(nbytes, us):
         return nbytes / (us * 1e-6) / 1e9
 
-    bw = {
-        "prep_1_gbs": gbs(n0.sum() * dim * esize + 12 * n0.sum(), kern["prep_1_us"]),
-        "pair_average_1_gbs": gbs((n0.sum() + n1.sum()) * dim * esize + 12 * n0.sum(), kern["pair_average_1_us"]),
+    # Algorithmic bytes of the bandwidth kernels.  prep reads the tokens and
+    # writes a norm and a key reset per row; pair average reads every input
+    # row once, writes the merged rows and moves 12 bytes of keys, map and
+    # representative list per input row (the mutual scan's traffic, counted
+    # here); gather reads each merged row it needs and writes the grid, and
+    # with two insertions also reads both maps and writes the composed one.
+    nbytes = {
+        "prep_1": n0.sum() * dim * esize + 12 * n0.sum(),
+        "pair_average_1": (n0.sum() + n1.sum()) * dim * esize + 12 * n0.sum(),
     }
     if p.two:
-        bw["prep_2_gbs"] = gbs(n1.sum() * dim * esize + 12 * n1.sum(), kern["prep_2_us"])
-        bw["pair_average_2_gbs"] = gbs((n1.sum() + n2.sum()) * dim * esize + 12 * n1.sum(),
-                                       kern["pair_average_2_us"])
-    # Gather reads each merged row it needs and writes the grid; with two
-    # insertions it also reads both maps and writes the composed one.
-    bw["gather_gbs"] = gbs((n2.sum() + n0.sum()) * dim * esize + (12 if p.two else 4) * n0.sum(),
-                           kern["compose_gather_us" if p.two else "gather_us"])
+        nbytes["prep_2"] = n1.sum() * dim * esize + 12 * n1.sum()
+        nbytes["pair_average_2"] = (n1.sum() + n2.sum()) * dim * esize + 12 * n1.sum()
+    nbytes["gather"] = (n2.sum() + n0.sum()) * dim * esize + (12 if p.two else 4) * n0.sum()
+    kern_us = dict((k, kern[f"{k}_us"]) for k in nbytes if k != "gather")
+    kern_us["gather"] = kern["compose_gather_us" if p.two else "gather_us"]
+    bw = {f"{k}_gbs": gbs(v, kern_us[k]) for k, v in nbytes.items()}
     for k in list(bw):
         bw[k.replace("_gbs", "_frac")] = bw[k] / hbm
+    # The whole step against its roofline: the time the affinity flops need
+    # at the tensor peak plus the time the bandwidth kernels' bytes need at
+    # the copy bandwidth, over the measured step time.
+    flops_step = alg1 + alg2
+    bytes_step = float(sum(nbytes.values()))
+    tensor_us = flops_step / (burst * 1e12) * 1e6
+    hbm_us = bytes_step / (hbm * 1e9) * 1e6
+    pipeline = {"flops_per_step": flops_step, "bytes_per_step": bytes_step,
+                "tensor_us_at_peak": tensor_us, "hbm_us_at_peak": hbm_us,
+                "ideal_us": tensor_us + hbm_us, "measured_us": 1e3 * t["ms"],
+                "frac": (tensor_us + hbm_us) / (1e3 * t["ms"]),
+                "definition": "(algorithmic affinity flops / bf16 burst peak + algorithmic bytes of prep, "
+                              "pair average and gather / measured copy bandwidth) / step time"}
     return {"n0": n0, "n1": n1, "n2": n2, "alg1": alg1, "alg2": alg2,
             "aff_launches": len(aff_ms), "aff_flops_per_launch": sum(aff_flops) / len(aff_ms),
             "aff_tflops": achieved, "aff_peak_burst": burst, "aff_peak_sustained": sustained,
-            "aff_executed_tflops": executed, "hbm": bw, "hbm_peak": hbm,
+            "aff_executed_tflops": executed, "hbm": bw, "hbm_peak": hbm, "pipeline": pipeline,
             "rows_per_aff_launch": (n0.sum() + (n1.sum() if p.two else 0.0)) / (2.0 if p.two else 1.0)}
 
 
@@ -539,6 +557,7 @@ def workload_summary(p: Step, t: dict, m: dict) -> dict:
         "affinity_peak": ("bf16 dense" if p.cfg.dtype == "bf16" else
                           "tf32 dense = bf16 x 1.1/2.25 (nominal ratio); three tf32 products per term"),
         "affinity_us": {k: v for k, v in t["kern"].items() if k.startswith("affinity")},
+        "pipeline_frac": m["pipeline"]["frac"],
     }
     out.update({k: v for k, v in m["hbm"].items() if k.endswith("_frac")})
     return out
@@ -840,6 +859,7 @@ def run_mpm(args):
             "merged_tokens": {"stage0": int(n0.sum()), "stage1": int(n1.sum()), "stage2": int(n2.sum())},
             "roofline": roofline,
             "hbm_kernels": hbm_kernels,
+            "pipeline_roofline": m["pipeline"],
             "per_workload": per_workload,
             "padded_batch": padded,
             "chunked_similarity": chunked,

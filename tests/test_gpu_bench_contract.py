@@ -45,7 +45,13 @@ def test_gpu_arm_prints_one_contract_line():
         assert w["images_per_s"] > 0 and w["tokens_per_s"] > 0, name
         assert 0 < w["affinity_frac_of_burst"] < 1.5 and 0 < w["gather_frac"] < 1.5, name
         assert 0 < w["pair_average_1_frac"] < 1.5 and 0 < w["prep_1_frac"] < 1.5, name
+        assert 0 < w["pipeline_frac"] < 1.5, name
     assert abs(pw["vit_b"]["images_per_s"] - d["value"]) < 1e-6 * d["value"]
+    # The whole step against its combined tensor + HBM roofline.
+    pr = d["pipeline_roofline"]
+    assert abs(pr["ideal_us"] - pr["tensor_us_at_peak"] - pr["hbm_us_at_peak"]) < 1e-9 * pr["ideal_us"]
+    assert abs(pr["frac"] - pr["ideal_us"] / pr["measured_us"]) < 1e-9 and 0 < pr["frac"] < 1.5
+    assert abs(pr["measured_us"] - 1e3 * d["ms_per_step"]) < 1e-6 * pr["measured_us"]
     # The in-step timeline of the traced library, beside the event figures.
     ins = d["in_step"]
     assert ins is not None and ins["affinity_tflops_algorithmic"] > 0
