@@ -544,14 +544,25 @@ __global__ void __launch_bounds__(Epi<EPIW>::THREADS, 1)
 #pragma unroll
       for (int h = 0; h < EPI_COLS / 32; ++h) colcand[h] = 0ull;
       const uint32_t taddr = tmem + lane_addr + static_cast<uint32_t>(acc * TILE + c0);
-      if (diag) {
+      if constexpr (EPI_COLS > 64) {
+        // Column candidates go to the keys inside the slice loop.
+        unsigned long long* const colkeys = ws.keys + it.base + it.col0 + c0 + lane;
+        if (diag) {
+          epilogue_slice_rolled<EPI_COLS, true, false>(taddr, sc, c0, jd, best, bj, inv_i, lane, row_base, it.n,
+                                                       it.col0, it.origin, scr, colkeys);
+        } else if (col_update) {
+          epilogue_slice_rolled<EPI_COLS, false, true>(taddr, sc, c0, jd, best, bj, inv_i, lane, row_base, it.n,
+                                                       it.col0, it.origin, scr, colkeys);
+        }
+      } else if (diag) {
         epilogue_slice<EPI_COLS, true, false>(taddr, sc, c0, jd, best, bj, inv_i, lane, row_base, it.n, it.col0,
                                               it.origin, scr, colcand);
       } else if (col_update) {
         epilogue_slice<EPI_COLS, false, true>(taddr, sc, c0, jd, best, bj, inv_i, lane, row_base, it.n, it.col0,
                                               it.origin, scr, colcand);
       }
-      // Release the accumulator first, then merge this tile's candidates.
+      // Release the accumulator first, then merge this tile's candidates
+      // (the rolled slice has merged its column candidates already).
       ptx::tc_fence_before_sync();
       if (leader) {
         ptx::mbar_arrive(&ctl->acc_empty[acc]);
