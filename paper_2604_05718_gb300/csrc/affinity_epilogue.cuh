@@ -166,31 +166,30 @@ __device__ __forceinline__ void epilogue_slice(uint32_t taddr, const float* sc, 
   }
 }
 
-// The same slice with the 32-column loop left rolled, for 128-column
-// slices, whose unrolled code is twice as long: the column candidate of
-// tile column c0 + 32 h + lane goes straight to colkeys[32 h] (colkeys
-// points at this lane's first column) instead of a register array, which
-// would need the loop unrolled.  (Measured on vit_b: step 0.2051-0.2054
+// The same slice with the 32-column loop left rolled (`steps` steps of 32
+// columns), for 128-column slices, whose unrolled code is twice as long:
+// the column candidate of tile column c0 + 32 h + lane goes straight to
+// colkeys[32 h] (colkeys points at this lane's first column) instead of a
+// register array, which would need the loop unrolled.  (Measured on vit_b: step 0.2051-0.2054
 // against 0.2069-0.2073 ms unrolled; the 64-column slices of the 16-warp
 // epilogue stay unrolled, where the rolled loop was 1.4% slower.)
-template <int COLS, bool DIAG, bool COL>
+template <bool DIAG, bool COL>
 __device__ __forceinline__ void epilogue_slice_rolled(uint32_t taddr, const float* sc, int c0, int jd, float& best,
                                                       int& bj, float inv_i, int lane, int row_base, int n,
                                                       int col0, int origin, uint2* scratch,
-                                                      unsigned long long* colkeys) {
-  static_assert(COLS % 32 == 0, "slices are whole 32-column pairs of pieces");
+                                                      unsigned long long* colkeys, int steps) {
   float best0 = -INFINITY, best1 = -INFINITY;
   int bj0 = -1, bj1 = -1;
   uint32_t va[16], vb[16];
   ptx::tmem_ld_32x32b_x16(taddr, va);
   ptx::tmem_wait_ld(va);
 #pragma unroll 1
-  for (int h = 0; h < COLS / 32; ++h) {
+  for (int h = 0; h < steps; ++h) {
     const int c = c0 + 32 * h;
     ptx::tmem_ld_32x32b_x16(taddr + 32 * h + 16, vb);
     epilogue_piece<DIAG, COL>(va, sc, c, jd, best0, bj0, best1, bj1, inv_i, lane, scratch, 0);
     ptx::tmem_wait_ld(vb);
-    const bool more = h + 1 < COLS / 32;
+    const bool more = h + 1 < steps;
     if (more) ptx::tmem_ld_32x32b_x16(taddr + 32 * h + 32, va);
     epilogue_piece<DIAG, COL>(vb, sc, c + 16, jd, best0, bj0, best1, bj1, inv_i, lane, scratch, 16);
     if (COL) {

@@ -26,6 +26,14 @@
 //    thread's 128-row block also yields column candidates (row j scores row
 //    i by G_ij / |x_i|), as in affinity_tc.cu's symmetric mode; the block
 //    below the diagonal of a diagonal tile is skipped.
+//  * A tile whose column block holds at most 128 columns of its chunk (the
+//    last block of a ragged image: 94 of 256 for an image of 862 tokens) is
+//    narrow: its MMAs run with N = 128, each CTA staging 64 of its B rows,
+//    and the 8-warp epilogue splits its 128 accumulator columns between
+//    both column halves of warps.  The MMA warp picks the tile shape once
+//    per tile, from a bit set while the items were decoded, and issues the
+//    tile's stages with compile-time instruction descriptors: a descriptor
+//    chosen at run time slowed every tile's issue.
 //
 // Rows of the tile are assigned crosswise: the leader CTA (rank 0, whose
 // warp 1 issues the MMAs) holds tile rows [128, 256) and the peer rows
@@ -46,6 +54,7 @@
 #include <math.h>
 
 #include <atomic>
+#include <type_traits>
 
 #include "mpm.h"
 #include "affinity_epilogue.cuh"
@@ -81,12 +90,16 @@ struct Epi {
 constexpr int kWideEpilogueMaxDim = 512;  // bf16 rows of at most this many features take 16 epilogue warps
 constexpr uint32_t TMEM_COLS = 2 * TILE;
 constexpr uint32_t IDESC = ptx::idesc_bf16_f32(2 * HALF, TILE);
+// Narrow tiles (at most HALF columns of the tile inside the chunk) run
+// N = HALF MMAs: half the tensor work, and each CTA holds HALF / 2 B rows.
+constexpr uint32_t IDESC_NARROW = ptx::idesc_bf16_f32(2 * HALF, HALF);
 // fp32 tokens: three tf32 products per K slice (hi hi + hi lo + lo hi, the
 // "3xTF32" split), with a stage of 32 features holding four 16 KiB slices:
 // A high, A low, B high, B low (one 128-byte swizzle row of fp32 each).
 constexpr int TF_BOX_K = 32;
 constexpr int TF_BK = TF_BOX_K;
 constexpr uint32_t IDESC_TF32 = ptx::idesc_tf32_f32(2 * HALF, TILE);
+constexpr uint32_t IDESC_TF32_NARROW = ptx::idesc_tf32_f32(2 * HALF, HALF);
 static_assert(4 * ATOM_BYTES == STAGE_BYTES && HALF * TF_BOX_K * 4 == ATOM_BYTES, "same stage size for both paths");
 constexpr uint64_t WAIT_LIMIT_NS = 2000000000ull;
 constexpr int kMaxItems = 160;
@@ -98,6 +111,7 @@ struct Control {
   uint64_t acc_full[2];         // both: accumulator a complete
   uint64_t acc_empty[2];        // leader: both CTAs finished reading accumulator a
   uint64_t drain;               // leader: all MMAs completed
+  uint32_t narrow_bits[(kMaxItems + 31) / 32];  // bit k: this cluster's item k is narrow
   uint32_t tmem_base;
   int abort_flag;
 };
@@ -146,6 +160,17 @@ __device__ __forceinline__ Item decode_pair_item(const int64_t* plan, const int6
   it.row0 = static_cast<int>(lo) * TILE;
   it.col0 = static_cast<int>(lo + local) * TILE;
   return it;
+}
+
+// At most HALF columns of the tile lie in its chunk: the last column block
+// of a ragged image, e.g. 94 of 256 for an image of 862 tokens.
+__device__ __forceinline__ bool is_narrow(const Item& it) { return it.n - it.col0 <= HALF; }
+
+// Whether item w is narrow, for items past the shared-memory list (out of
+// line: the MMA warp's loop stays small).
+__device__ __noinline__ bool narrow_item_slow(const int64_t* plan, const int64_t* soff, int batch, int64_t w,
+                                              int64_t chunk) {
+  return is_narrow(decode_pair_item(plan, soff, batch, w, chunk));
 }
 
 __device__ __forceinline__ uint32_t cluster_rank() {
@@ -369,8 +394,18 @@ __global__ void __launch_bounds__(Epi<EPIW>::THREADS, 1)
   const int64_t* soff = staged ? soff_s : ws.soff;
   const int64_t total = plan[batch];
   const int64_t count = total > cid ? (total - 1 - cid) / clusters + 1 : 0;
-  for (int64_t k = threadIdx.x; k < count && k < kMaxItems; k += THREADS)
-    items[k] = decode_pair_item(plan, soff, batch, cid + k * clusters, chunk);
+  static_assert(THREADS >= kMaxItems, "one thread decodes each listed item");
+  {
+    const int k = threadIdx.x;
+    bool nb = false;
+    if (k < count && k < kMaxItems) {
+      items[k] = decode_pair_item(plan, soff, batch, cid + k * clusters, chunk);
+      nb = is_narrow(items[k]);
+    }
+    // The MMA warp reads one bit per item instead of the item.
+    const uint32_t bits = __ballot_sync(0xFFFFFFFFu, nb);
+    if ((k & 31) == 0 && k < kMaxItems) ctl->narrow_bits[k >> 5] = bits;
+  }
   __syncthreads();
   auto item = [&](int64_t k) -> Item {
     return k < kMaxItems ? items[k] : decode_pair_item(plan, soff, batch, cid + k * clusters, chunk);
@@ -388,7 +423,7 @@ __global__ void __launch_bounds__(Epi<EPIW>::THREADS, 1)
       for (int64_t k = 0; ok && k < count; ++k) {
         const Item it = item(k);
         const int32_t arow = static_cast<int32_t>(it.base + it.row0 + HALF * (rank ^ 1u));
-        const int32_t brow = static_cast<int32_t>(it.base + it.col0 + HALF * rank);
+        const int32_t brow = static_cast<int32_t>(it.base + it.col0 + (is_narrow(it) ? HALF / 2 : HALF) * rank);
         for (int kb = 0; kb < ksteps; ++kb) {
           if (!ptx::mbar_wait(&ctl->empty[stage], phase ^ 1u, abort_flag, WAIT_LIMIT_NS)) {
             fail(ctl, ws.status, 11);
@@ -440,44 +475,61 @@ __global__ void __launch_bounds__(Epi<EPIW>::THREADS, 1)
         }
         ptx::tc_fence_after_sync();
         const uint32_t d_tmem = tmem + static_cast<uint32_t>(acc * TILE);
-        for (int kb = 0; kb < ksteps; ++kb) {
-          if (!ptx::mbar_wait(&ctl->full[stage], phase, abort_flag, WAIT_LIMIT_NS)) {
-            fail(ctl, ws.status, 13);
-            ok = false;
-            break;
-          }
-          ptx::tc_fence_after_sync();
-          const uint64_t a_desc = desc0 + static_cast<uint64_t>((stage * STAGE_BYTES) >> 4);
-          if constexpr (TF32) {
-            if ((kb + 1) * kBK <= dim) {
-              mma_stage_tf32x3(d_tmem, a_desc, IDESC_TF32, kb != 0 ? 1u : 0u, &ctl->empty[stage]);
+        const bool narrow = k < kMaxItems ? ((ctl->narrow_bits[k >> 5] >> (k & 31)) & 1u) != 0u
+                                          : narrow_item_slow(plan, soff, batch, cid + k * clusters, chunk);
+        // One tile's stages, with its instruction descriptors as compile-time
+        // constants (ID, ID_TF32): the tile shape is chosen once per tile,
+        // outside the stage loop, so no descriptor is a run-time value.
+        auto issue_tile = [&](auto id, auto id_tf32) {
+          constexpr uint32_t ID = decltype(id)::value;
+          constexpr uint32_t ID_TF32 = decltype(id_tf32)::value;
+          for (int kb = 0; kb < ksteps; ++kb) {
+            if (!ptx::mbar_wait(&ctl->full[stage], phase, abort_flag, WAIT_LIMIT_NS)) {
+              fail(ctl, ws.status, 13);
+              ok = false;
+              break;
+            }
+            ptx::tc_fence_after_sync();
+            const uint64_t a_desc = desc0 + static_cast<uint64_t>((stage * STAGE_BYTES) >> 4);
+            if constexpr (TF32) {
+              if ((kb + 1) * kBK <= dim) {
+                mma_stage_tf32x3(d_tmem, a_desc, ID_TF32, kb != 0 ? 1u : 0u, &ctl->empty[stage]);
+              } else {
+                // Last, partial stage: the K = 8 slices that hold features.
+                for (int kk = 0; kk < kBK / 8 && kb * kBK + kk * 8 < dim; ++kk) {
+                  const uint64_t ah = a_desc + 2 * kk, al = ah + (ATOM_BYTES >> 4);
+                  const uint64_t bh = ah + 2 * (ATOM_BYTES >> 4), bl = ah + 3 * (ATOM_BYTES >> 4);
+                  mma_pair_tf32(d_tmem, ah, bh, ID_TF32, (kb | kk) != 0 ? 1u : 0u);
+                  mma_pair_tf32(d_tmem, ah, bl, ID_TF32, 1u);
+                  mma_pair_tf32(d_tmem, al, bh, ID_TF32, 1u);
+                }
+                commit_both(&ctl->empty[stage]);
+              }
+            } else if ((kb + 1) * BK <= dim) {
+              mma_stage_full(d_tmem, a_desc, ID, kb != 0 ? 1u : 0u, &ctl->empty[stage]);
             } else {
-              // Last, partial stage: the K = 8 slices that hold features.
-              for (int kk = 0; kk < kBK / 8 && kb * kBK + kk * 8 < dim; ++kk) {
-                const uint64_t ah = a_desc + 2 * kk, al = ah + (ATOM_BYTES >> 4);
-                const uint64_t bh = ah + 2 * (ATOM_BYTES >> 4), bl = ah + 3 * (ATOM_BYTES >> 4);
-                mma_pair_tf32(d_tmem, ah, bh, IDESC_TF32, (kb | kk) != 0 ? 1u : 0u);
-                mma_pair_tf32(d_tmem, ah, bl, IDESC_TF32, 1u);
-                mma_pair_tf32(d_tmem, al, bh, IDESC_TF32, 1u);
+              // Last, partial stage: only the K slices that hold features.
+              for (int kk = 0; kk < BK / 16 && kb * BK + kk * 16 < dim; ++kk) {
+                // K = 16 slice kk: swizzle atom kk / 4, 32 bytes per slice within it.
+                const uint64_t off = static_cast<uint64_t>((kk / 4) * (ATOM_BYTES >> 4) + (kk % 4) * 2);
+                mma_pair(d_tmem, a_desc + off, a_desc + (SLICE_BYTES >> 4) + off, ID, (kb | kk) != 0 ? 1u : 0u);
               }
               commit_both(&ctl->empty[stage]);
             }
-          } else if ((kb + 1) * BK <= dim) {
-            mma_stage_full(d_tmem, a_desc, IDESC, kb != 0 ? 1u : 0u, &ctl->empty[stage]);
-          } else {
-            // Last, partial stage: only the K slices that hold features.
-            for (int kk = 0; kk < BK / 16 && kb * BK + kk * 16 < dim; ++kk) {
-              // K = 16 slice kk: swizzle atom kk / 4, 32 bytes per slice within it.
-              const uint64_t off = static_cast<uint64_t>((kk / 4) * (ATOM_BYTES >> 4) + (kk % 4) * 2);
-              mma_pair(d_tmem, a_desc + off, a_desc + (SLICE_BYTES >> 4) + off, IDESC, (kb | kk) != 0 ? 1u : 0u);
+            if (++stage == STAGES) {
+              stage = 0;
+              phase ^= 1u;
             }
-            commit_both(&ctl->empty[stage]);
           }
-          if (++stage == STAGES) {
-            stage = 0;
-            phase ^= 1u;
-          }
-        }
+        };
+        using NarrowId = std::integral_constant<uint32_t, IDESC_NARROW>;
+        using NarrowIdTf32 = std::integral_constant<uint32_t, IDESC_TF32_NARROW>;
+        using FullId = std::integral_constant<uint32_t, IDESC>;
+        using FullIdTf32 = std::integral_constant<uint32_t, IDESC_TF32>;
+        if (narrow)
+          issue_tile(NarrowId{}, NarrowIdTf32{});
+        else
+          issue_tile(FullId{}, FullIdTf32{});
         if (!ok) break;
         commit_both(&ctl->acc_full[acc]);
         if (++acc == 2) {
@@ -492,21 +544,26 @@ __global__ void __launch_bounds__(Epi<EPIW>::THREADS, 1)
   } else {
     // ---------------- epilogue (both CTAs) ----------------
     // Warp (q, quarter) reads tile rows 32q..32q+31 of this CTA and tile
-    // columns c0..c0+EPI_COLS-1.  It keeps its own copy of those column
-    // scales, so no epilogue warp ever waits for another one.
+    // columns c0..c0+EPI_COLS-1, c0 = quarter * EPI_COLS.  A narrow tile's
+    // accumulator holds HALF columns: the 8-warp epilogue splits them
+    // between its two quarters (HALF / 2 each), and the 16-warp one leaves
+    // its upper two quarters idle.  Each warp keeps its own copy of its
+    // column scales, so no epilogue warp ever waits for another one.
     const int ew = warp - 2;
     const int q = warp & 3;
     const int quarter = ew >> 2;
     const uint32_t lane_addr = static_cast<uint32_t>(q * 32) << 16;
-    const int c0 = quarter * EPI_COLS;
+    auto first_col = [&](const Item& t) {
+      return (EPI_WARPS == 8 && is_narrow(t)) ? quarter * (HALF / 2) : quarter * EPI_COLS;
+    };
     float* my_scale = scale + ew * EPI_COLS;
-    const float* sc = my_scale - c0;  // indexed by tile column
     uint2* scr = scratch_all + ew * 32;
     int acc = 0;
     uint32_t acc_phase = 0;
     float pf_scale[EPI_COLS / 32], pf_inv = 0.f;
     auto prefetch = [&](const Item& nx) {
       const float nan = __int_as_float(0x7fc00000);  // columns outside the image never win
+      const int c0 = first_col(nx);
 #pragma unroll
       for (int h = 0; h < EPI_COLS / 32; ++h) {
         const int j = nx.col0 + c0 + 32 * h + lane;
@@ -531,13 +588,17 @@ __global__ void __launch_bounds__(Epi<EPIW>::THREADS, 1)
       }
       if (k + 1 < count) prefetch(item(k + 1));
       ptx::tc_fence_after_sync();
+      const bool narrow = is_narrow(it);
+      const int c0 = first_col(it);
+      const float* sc = my_scale - c0;  // indexed by tile column
       const int row_base = it.row0 + HALF * static_cast<int>(rank ^ 1u) + q * 32;
       const int row = row_base + lane;
       const int jd = row - it.col0;
       const int iblk = (it.row0 + HALF * static_cast<int>(rank ^ 1u)) / HALF;
       const int jblk = (it.col0 + c0) / HALF;
-      const bool diag = jblk == iblk;
-      const bool col_update = jblk > iblk;
+      const bool live = !narrow || c0 < HALF;  // inside the narrow accumulator
+      const bool diag = live && jblk == iblk;
+      const bool col_update = live && jblk > iblk;
       float best = -INFINITY;
       int bj = -1;
       unsigned long long colcand[EPI_COLS / 32];
@@ -547,12 +608,13 @@ __global__ void __launch_bounds__(Epi<EPIW>::THREADS, 1)
       if constexpr (EPI_COLS > 64) {
         // Column candidates go to the keys inside the slice loop.
         unsigned long long* const colkeys = ws.keys + it.base + it.col0 + c0 + lane;
+        const int steps = narrow ? HALF / 2 / 32 : EPI_COLS / 32;
         if (diag) {
-          epilogue_slice_rolled<EPI_COLS, true, false>(taddr, sc, c0, jd, best, bj, inv_i, lane, row_base, it.n,
-                                                       it.col0, it.origin, scr, colkeys);
+          epilogue_slice_rolled<true, false>(taddr, sc, c0, jd, best, bj, inv_i, lane, row_base, it.n, it.col0,
+                                             it.origin, scr, colkeys, steps);
         } else if (col_update) {
-          epilogue_slice_rolled<EPI_COLS, false, true>(taddr, sc, c0, jd, best, bj, inv_i, lane, row_base, it.n,
-                                                       it.col0, it.origin, scr, colkeys);
+          epilogue_slice_rolled<false, true>(taddr, sc, c0, jd, best, bj, inv_i, lane, row_base, it.n, it.col0,
+                                             it.origin, scr, colkeys, steps);
         }
       } else if (diag) {
         epilogue_slice<EPI_COLS, true, false>(taddr, sc, c0, jd, best, bj, inv_i, lane, row_base, it.n, it.col0,
