@@ -492,12 +492,17 @@ def step_metrics(p: Step, t: dict, peaks: dict, peak_kind: str) -> dict:
     burst = ratio * peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
     sustained = ratio * peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
     # What the tensor pipe executes (bf16): the 256 x 256 tiles on or above
-    # each image's diagonal, over K padded to 16 (the MMA's K).
+    # each image's diagonal, over K padded to 16 (the MMA's K).  The R tiles
+    # of an image's last column block are narrow (256 x 128) when that block
+    # holds at most 128 of its tokens.
     kpad = -(-dim // 16) * 16
 
     def exec_flops(ns):
-        r = -(-ns.astype(np.int64) // 256)
-        return float(np.sum(r * (r + 1) // 2)) * 256 * 256 * 2 * kpad
+        n = ns.astype(np.int64)
+        r = -(-n // 256)
+        narrow = (n > 0) & (n - 256 * (r - 1) <= 128)
+        tiles = r * (r + 1) / 2.0 - np.where(narrow, r / 2.0, 0.0)
+        return float(np.sum(tiles)) * 256 * 256 * 2 * kpad
 
     exe = [exec_flops(n0)] * len(t["aff_ms_1"]) + [exec_flops(n1)] * len(t["aff_ms_2"])
     executed = sum(exe) / (sum(aff_ms) * 1e-3) / 1e12 if cfg.dtype == "bf16" else None
@@ -643,7 +648,8 @@ def run_mpm(args):
         "executed_tflops": m["aff_executed_tflops"],
         "executed_frac": (m["aff_executed_tflops"] / m["aff_peak_burst"]
                           if m["aff_executed_tflops"] is not None else None),
-        "executed_definition": "MMA work issued: 256x256 tiles on or above the diagonal x K padded to 16",
+        "executed_definition": ("MMA work issued: 256x256 tiles on or above the diagonal (256x128 where the "
+                                "column block holds at most 128 tokens) x K padded to 16"),
         "traffic": traffic_for(AFFINITY_SOURCES, m["rows_per_aff_launch"]),
     }
     hbm_kernels = dict(m["hbm"], peak_gbs=m["hbm_peak"], peak_kind=f"{peak_kind} copy bandwidth")

@@ -58,8 +58,31 @@ def test_affinity_flops_and_rate(bench):
     # Two launches of each stage: (2 * 144 + 2 * 64) flops in 6 us.
     assert m["aff_tflops"] == pytest.approx(416.0 / 6e-6 / 1e12, rel=1e-12)
     assert m["aff_peak_burst"] == 1000.0 and m["aff_peak_sustained"] == 800.0
-    # Executed: every image is one 256 x 256 tile, K padded to 16.
-    assert m["aff_executed_tflops"] == pytest.approx(4 * 2 * 256 * 256 * 2 * 16 / 6e-6 / 1e12, rel=1e-12)
+    # Executed: every image is one tile whose column block holds at most 128
+    # tokens, so a narrow 256 x 128 one; K padded to 16.
+    assert m["aff_executed_tflops"] == pytest.approx(4 * 2 * 256 * 128 * 2 * 16 / 6e-6 / 1e12, rel=1e-12)
+
+
+def test_executed_tiles_count_narrow_ones_at_half_width(bench):
+    # 862 tokens: R = 4, last block 94 tokens, so its 4 tiles are narrow:
+    # 10 - 4 / 2 = 8 full-tile equivalents; 1024 tokens: 10 full tiles;
+    # 1100 tokens: R = 5, last block 76: 15 - 5 / 2 = 12.5.
+    class Cfg:
+        dim, dtype, insertions = 768, "bf16", 1
+
+    class Batch:
+        offsets = np.array([0, 862, 1886, 2986])
+        batch, rows = 3, 2986
+
+    class Step:
+        cfg, batch, two = Cfg, Batch, False
+        off1_h = np.array([0, 862, 1886, 2986])
+        off2 = None
+
+    t = {"ms": 0.1, "kern": {"prep_1_us": 1.0, "pair_average_1_us": 1.0, "gather_us": 1.0},
+         "aff_ms_1": [0.001], "aff_ms_2": []}
+    m = bench.step_metrics(Step, t, PEAKS, "measured")
+    assert m["aff_executed_tflops"] == pytest.approx((8 + 10 + 12.5) * 256 * 256 * 2 * 768 / 1e-6 / 1e12, rel=1e-12)
 
 
 def test_bandwidth_kernel_bytes(bench):
