@@ -481,8 +481,8 @@ __global__ void __launch_bounds__(Epi<EPIW>::THREADS, 1)
         // constants (ID, ID_TF32): the tile shape is chosen once per tile,
         // outside the stage loop, so no descriptor is a run-time value.
         auto issue_tile = [&](auto id, auto id_tf32) {
-          constexpr uint32_t ID = decltype(id)::value;
-          constexpr uint32_t ID_TF32 = decltype(id_tf32)::value;
+          [[maybe_unused]] constexpr uint32_t ID = decltype(id)::value;            // bf16 instances
+          [[maybe_unused]] constexpr uint32_t ID_TF32 = decltype(id_tf32)::value;  // tf32 instance
           for (int kb = 0; kb < ksteps; ++kb) {
             if (!ptx::mbar_wait(&ctl->full[stage], phase, abort_flag, WAIT_LIMIT_NS)) {
               fail(ctl, ws.status, 13);
