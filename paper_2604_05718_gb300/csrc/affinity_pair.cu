@@ -166,11 +166,11 @@ __device__ __forceinline__ Item decode_pair_item(const int64_t* plan, const int6
 // of a ragged image, e.g. 94 of 256 for an image of 862 tokens.
 __device__ __forceinline__ bool is_narrow(const Item& it) { return it.n - it.col0 <= HALF; }
 
-// Whether item w is narrow, for items past the shared-memory list (out of
-// line: the MMA warp's loop stays small).
-__device__ __noinline__ bool narrow_item_slow(const int64_t* plan, const int64_t* soff, int batch, int64_t w,
+// Item w, for items past the shared-memory list: out of line, so that the
+// role loops that fall back on it stay small.
+__device__ __noinline__ Item decode_item_slow(const int64_t* plan, const int64_t* soff, int batch, int64_t w,
                                               int64_t chunk) {
-  return is_narrow(decode_pair_item(plan, soff, batch, w, chunk));
+  return decode_pair_item(plan, soff, batch, w, chunk);
 }
 
 __device__ __forceinline__ uint32_t cluster_rank() {
@@ -408,7 +408,7 @@ __global__ void __launch_bounds__(Epi<EPIW>::THREADS, 1)
   }
   __syncthreads();
   auto item = [&](int64_t k) -> Item {
-    return k < kMaxItems ? items[k] : decode_pair_item(plan, soff, batch, cid + k * clusters, chunk);
+    return k < kMaxItems ? items[k] : decode_item_slow(plan, soff, batch, cid + k * clusters, chunk);
   };
   volatile int* abort_flag = &ctl->abort_flag;
 
@@ -476,7 +476,7 @@ __global__ void __launch_bounds__(Epi<EPIW>::THREADS, 1)
         ptx::tc_fence_after_sync();
         const uint32_t d_tmem = tmem + static_cast<uint32_t>(acc * TILE);
         const bool narrow = k < kMaxItems ? ((ctl->narrow_bits[k >> 5] >> (k & 31)) & 1u) != 0u
-                                          : narrow_item_slow(plan, soff, batch, cid + k * clusters, chunk);
+                                          : is_narrow(decode_item_slow(plan, soff, batch, cid + k * clusters, chunk));
         // One tile's stages, with its instruction descriptors as compile-time
         // constants (ID, ID_TF32): the tile shape is chosen once per tile,
         // outside the stage loop, so no descriptor is a run-time value.
