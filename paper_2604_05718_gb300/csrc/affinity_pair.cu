@@ -30,7 +30,9 @@
 //    last block of a ragged image: 94 of 256 for an image of 862 tokens) is
 //    narrow: its MMAs run with N = 128, each CTA staging 64 of its B rows,
 //    and the 8-warp epilogue splits its 128 accumulator columns between
-//    both column halves of warps.  The MMA warp picks the tile shape once
+//    both column halves of warps.  With 8 epilogue warps, a last round of
+//    tiles that would leave half of the SM pairs idle is dealt as narrow
+//    256 x 128 halves instead.  The MMA warp picks the tile shape once
 //    per tile, from a bit set while the items were decoded, and issues the
 //    tile's stages with compile-time instruction descriptors: a descriptor
 //    chosen at run time slowed every tile's issue.
@@ -120,8 +122,9 @@ struct Item {
   int64_t base;  // global row of the first token of the tile's chunk
   int n;         // tokens in the chunk (the image without chunking)
   int row0;      // first row of the tile within the chunk (a multiple of 256)
-  int col0;      // first column of the tile within the chunk (a multiple of 256)
+  int col0;      // first column of the tile within the chunk (a multiple of 128)
   int origin;    // index of the chunk's first token within its image
+  int narrow;    // 1: a 256 x 128 tile (N = 128 MMAs) of columns col0 .. col0 + 127
 };
 
 template <int EPIW>
@@ -159,18 +162,34 @@ __device__ __forceinline__ Item decode_pair_item(const int64_t* plan, const int6
   local -= lo * r - lo * (lo - 1) / 2;
   it.row0 = static_cast<int>(lo) * TILE;
   it.col0 = static_cast<int>(lo + local) * TILE;
+  // At most HALF columns of the tile lie in its chunk: the last column block
+  // of a ragged image, e.g. 94 of 256 for an image of 862 tokens.
+  it.narrow = it.n - it.col0 <= HALF ? 1 : 0;
   return it;
 }
 
-// At most HALF columns of the tile lie in its chunk: the last column block
-// of a ragged image, e.g. 94 of 256 for an image of 862 tokens.
-__device__ __forceinline__ bool is_narrow(const Item& it) { return it.n - it.col0 <= HALF; }
+__device__ __forceinline__ bool is_narrow(const Item& it) { return it.narrow != 0; }
+
+// Item w of the launch.  The plan's tiles go to the SM pairs round-robin;
+// when the last round (tiles split_from .. total - 1) would leave at least
+// half of the pairs idle, each of its tiles is dealt as two 256 x 128
+// halves instead (items split_from + 2 t and split_from + 2 t + 1), so that
+// the round takes one narrow tile's time.
+__device__ __forceinline__ Item decode_launch_item(const int64_t* plan, const int64_t* soff, int batch, int64_t w,
+                                                   int64_t chunk, int64_t split_from) {
+  if (w < split_from) return decode_pair_item(plan, soff, batch, w, chunk);
+  const int64_t h = w - split_from;
+  Item it = decode_pair_item(plan, soff, batch, split_from + (h >> 1), chunk);
+  if (h & 1) it.col0 += HALF;
+  it.narrow = 1;
+  return it;
+}
 
 // Item w, for items past the shared-memory list: out of line, so that the
 // role loops that fall back on it stay small.
 __device__ __noinline__ Item decode_item_slow(const int64_t* plan, const int64_t* soff, int batch, int64_t w,
-                                              int64_t chunk) {
-  return decode_pair_item(plan, soff, batch, w, chunk);
+                                              int64_t chunk, int64_t split_from) {
+  return decode_launch_item(plan, soff, batch, w, chunk, split_from);
 }
 
 __device__ __forceinline__ uint32_t cluster_rank() {
@@ -392,14 +411,20 @@ __global__ void __launch_bounds__(Epi<EPIW>::THREADS, 1)
   }
   const int64_t* plan = staged ? plan_s : ws.plan;
   const int64_t* soff = staged ? soff_s : ws.soff;
-  const int64_t total = plan[batch];
+  // A split last round pays only with 8 epilogue warps, whose column halves
+  // share a narrow tile's columns; the 16-warp epilogue reads 64 columns per
+  // warp for a half tile as for a full one (vit_s stage 2: 1 us slower).
+  const int64_t tiles = plan[batch];
+  const int64_t rest = tiles % clusters;
+  const int64_t split_from = (EPI_WARPS == 8 && rest > 0 && 2 * rest <= clusters) ? tiles - rest : tiles;
+  const int64_t total = tiles + (tiles - split_from);  // items: the split tiles count twice
   const int64_t count = total > cid ? (total - 1 - cid) / clusters + 1 : 0;
   static_assert(THREADS >= kMaxItems, "one thread decodes each listed item");
   {
     const int k = threadIdx.x;
     bool nb = false;
     if (k < count && k < kMaxItems) {
-      items[k] = decode_pair_item(plan, soff, batch, cid + k * clusters, chunk);
+      items[k] = decode_launch_item(plan, soff, batch, cid + k * clusters, chunk, split_from);
       nb = is_narrow(items[k]);
     }
     // The MMA warp reads one bit per item instead of the item.
@@ -408,7 +433,7 @@ __global__ void __launch_bounds__(Epi<EPIW>::THREADS, 1)
   }
   __syncthreads();
   auto item = [&](int64_t k) -> Item {
-    return k < kMaxItems ? items[k] : decode_item_slow(plan, soff, batch, cid + k * clusters, chunk);
+    return k < kMaxItems ? items[k] : decode_item_slow(plan, soff, batch, cid + k * clusters, chunk, split_from);
   };
   volatile int* abort_flag = &ctl->abort_flag;
 
@@ -476,7 +501,8 @@ __global__ void __launch_bounds__(Epi<EPIW>::THREADS, 1)
         ptx::tc_fence_after_sync();
         const uint32_t d_tmem = tmem + static_cast<uint32_t>(acc * TILE);
         const bool narrow = k < kMaxItems ? ((ctl->narrow_bits[k >> 5] >> (k & 31)) & 1u) != 0u
-                                          : is_narrow(decode_item_slow(plan, soff, batch, cid + k * clusters, chunk));
+                                          : is_narrow(decode_item_slow(plan, soff, batch, cid + k * clusters, chunk,
+                                                                       split_from));
         // One tile's stages, with its instruction descriptors as compile-time
         // constants (ID, ID_TF32): the tile shape is chosen once per tile,
         // outside the stage loop, so no descriptor is a run-time value.
