@@ -32,7 +32,8 @@
 //    and the 8-warp epilogue splits its 128 accumulator columns between
 //    both column halves of warps.  With 8 epilogue warps, a last round of
 //    tiles that would leave half of the SM pairs idle is dealt as narrow
-//    256 x 128 halves instead.  The MMA warp picks the tile shape once
+//    256 x 128 halves instead; a launch of at most 38 tiles (half of the 76
+//    SM pairs) is all last round, so each of its tiles is split.  The MMA warp picks the tile shape once
 //    per tile, from a bit set while the items were decoded, and issues the
 //    tile's stages with compile-time instruction descriptors: a descriptor
 //    chosen at run time slowed every tile's issue.
