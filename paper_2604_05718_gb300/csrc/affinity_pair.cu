@@ -336,6 +336,30 @@ __device__ __forceinline__ void commit_local(uint64_t* bar) {
                : "memory");
 }
 
+// Last, partial stage of a tile (the K slices that hold features), out of
+// line: it runs only when D is not a multiple of the stage width, and the
+// MMA warp's loop stays small.
+__device__ __noinline__ void mma_partial_stage_bf16(uint32_t d_tmem, uint64_t a_desc, uint32_t idesc, int kb,
+                                                    int dim, uint64_t* release) {
+  for (int kk = 0; kk < BK / 16 && kb * BK + kk * 16 < dim; ++kk) {
+    // K = 16 slice kk: swizzle atom kk / 4, 32 bytes per slice within it.
+    const uint64_t off = static_cast<uint64_t>((kk / 4) * (ATOM_BYTES >> 4) + (kk % 4) * 2);
+    mma_pair(d_tmem, a_desc + off, a_desc + (SLICE_BYTES >> 4) + off, idesc, (kb | kk) != 0 ? 1u : 0u);
+  }
+  commit_both(release);
+}
+__device__ __noinline__ void mma_partial_stage_tf32(uint32_t d_tmem, uint64_t a_desc, uint32_t idesc, int kb,
+                                                    int dim, uint64_t* release) {
+  for (int kk = 0; kk < TF_BK / 8 && kb * TF_BK + kk * 8 < dim; ++kk) {
+    const uint64_t ah = a_desc + 2 * kk, al = ah + (ATOM_BYTES >> 4);
+    const uint64_t bh = ah + 2 * (ATOM_BYTES >> 4), bl = ah + 3 * (ATOM_BYTES >> 4);
+    mma_pair_tf32(d_tmem, ah, bh, idesc, (kb | kk) != 0 ? 1u : 0u);
+    mma_pair_tf32(d_tmem, ah, bl, idesc, 1u);
+    mma_pair_tf32(d_tmem, al, bh, idesc, 1u);
+  }
+  commit_both(release);
+}
+
 __device__ __forceinline__ void fail(Control* ctl, int32_t* status, int32_t role) {
   ctl->abort_flag = 1;
   report(status, MPM_ERR_DEVICE_TIMEOUT, role);
@@ -522,26 +546,12 @@ __global__ void __launch_bounds__(Epi<EPIW>::THREADS, 1)
               if ((kb + 1) * kBK <= dim) {
                 mma_stage_tf32x3(d_tmem, a_desc, ID_TF32, kb != 0 ? 1u : 0u, &ctl->empty[stage]);
               } else {
-                // Last, partial stage: the K = 8 slices that hold features.
-                for (int kk = 0; kk < kBK / 8 && kb * kBK + kk * 8 < dim; ++kk) {
-                  const uint64_t ah = a_desc + 2 * kk, al = ah + (ATOM_BYTES >> 4);
-                  const uint64_t bh = ah + 2 * (ATOM_BYTES >> 4), bl = ah + 3 * (ATOM_BYTES >> 4);
-                  mma_pair_tf32(d_tmem, ah, bh, ID_TF32, (kb | kk) != 0 ? 1u : 0u);
-                  mma_pair_tf32(d_tmem, ah, bl, ID_TF32, 1u);
-                  mma_pair_tf32(d_tmem, al, bh, ID_TF32, 1u);
-                }
-                commit_both(&ctl->empty[stage]);
+                mma_partial_stage_tf32(d_tmem, a_desc, ID_TF32, kb, dim, &ctl->empty[stage]);
               }
             } else if ((kb + 1) * BK <= dim) {
               mma_stage_full(d_tmem, a_desc, ID, kb != 0 ? 1u : 0u, &ctl->empty[stage]);
             } else {
-              // Last, partial stage: only the K slices that hold features.
-              for (int kk = 0; kk < BK / 16 && kb * BK + kk * 16 < dim; ++kk) {
-                // K = 16 slice kk: swizzle atom kk / 4, 32 bytes per slice within it.
-                const uint64_t off = static_cast<uint64_t>((kk / 4) * (ATOM_BYTES >> 4) + (kk % 4) * 2);
-                mma_pair(d_tmem, a_desc + off, a_desc + (SLICE_BYTES >> 4) + off, ID, (kb | kk) != 0 ? 1u : 0u);
-              }
-              commit_both(&ctl->empty[stage]);
+              mma_partial_stage_bf16(d_tmem, a_desc, ID, kb, dim, &ctl->empty[stage]);
             }
             if (++stage == STAGES) {
               stage = 0;
