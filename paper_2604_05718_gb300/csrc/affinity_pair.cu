@@ -360,6 +360,18 @@ __device__ __noinline__ void mma_partial_stage_tf32(uint32_t d_tmem, uint64_t a_
   commit_both(release);
 }
 
+// Bounded wait for the producer and the epilogue: one probe inline, the
+// retry loop out of line, so that their loops stay small.  (The MMA warp
+// keeps ptx::mbar_wait inline: its waits are short and frequent.)
+__device__ __noinline__ bool mbar_wait_retry(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                             uint64_t limit_ns) {
+  return ptx::mbar_wait(bar, parity, abort_flag, limit_ns);
+}
+__device__ __forceinline__ bool mbar_wait_lean(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                               uint64_t limit_ns) {
+  return ptx::mbar_try_wait(bar, parity) || mbar_wait_retry(bar, parity, abort_flag, limit_ns);
+}
+
 __device__ __forceinline__ void fail(Control* ctl, int32_t* status, int32_t role) {
   ctl->abort_flag = 1;
   report(status, MPM_ERR_DEVICE_TIMEOUT, role);
@@ -475,7 +487,7 @@ __global__ void __launch_bounds__(Epi<EPIW>::THREADS, 1)
         const int32_t arow = static_cast<int32_t>(it.base + it.row0 + HALF * (rank ^ 1u));
         const int32_t brow = static_cast<int32_t>(it.base + it.col0 + (is_narrow(it) ? HALF / 2 : HALF) * rank);
         for (int kb = 0; kb < ksteps; ++kb) {
-          if (!ptx::mbar_wait(&ctl->empty[stage], phase ^ 1u, abort_flag, WAIT_LIMIT_NS)) {
+          if (!mbar_wait_lean(&ctl->empty[stage], phase ^ 1u, abort_flag, WAIT_LIMIT_NS)) {
             fail(ctl, ws.status, 11);
             ok = false;
             break;
@@ -619,7 +631,7 @@ __global__ void __launch_bounds__(Epi<EPIW>::THREADS, 1)
       for (int h = 0; h < EPI_COLS / 32; ++h) my_scale[32 * h + lane] = pf_scale[h];
       const float inv_i = pf_inv;
       __syncwarp();
-      if (!ptx::mbar_wait(&ctl->acc_full[acc], acc_phase, abort_flag, WAIT_LIMIT_NS)) {
+      if (!mbar_wait_lean(&ctl->acc_full[acc], acc_phase, abort_flag, WAIT_LIMIT_NS)) {
         fail(ctl, ws.status, 14);
         break;
       }
