@@ -7,9 +7,9 @@
 //
 //  * A cluster of two CTAs (an SM pair) computes a 256 x 256 tile of
 //    G = X X^T with tcgen05.mma.cta_group::2 (M = 256, N = 256).  CTA r holds
-//    tile rows [128r, 128r + 128) of A and tile columns [128r, 128r + 128) of
-//    B in its own shared memory, and receives its 128 rows x 256 columns of
-//    the accumulator in its own tensor memory.  Each SM therefore stages 64
+//    128 tile rows of A (assigned crosswise, below) and tile columns
+//    [128r, 128r + 128) of B in its own shared memory, and receives its 128
+//    rows x 256 columns of the accumulator in its own tensor memory.  Each SM therefore stages 64
 //    KiB per stage instead of 96 KiB, which leaves room for three stages and
 //    cuts the shared-memory traffic of the tensor cores by a third.
 //  * bf16 tokens: a stage holds 128 features (two 64-feature TMA boxes per
@@ -33,10 +33,11 @@
 //    both column halves of warps.  With 8 epilogue warps, a last round of
 //    tiles that would leave half of the SM pairs idle is dealt as narrow
 //    256 x 128 halves instead; a launch of at most 38 tiles (half of the 76
-//    SM pairs) is all last round, so each of its tiles is split.  The MMA warp picks the tile shape once
-//    per tile, from a bit set while the items were decoded, and issues the
-//    tile's stages with compile-time instruction descriptors: a descriptor
-//    chosen at run time slowed every tile's issue.
+//    SM pairs) is all last round, so each of its tiles is split.  The MMA
+//    warp picks the tile shape once per tile, from a bit set while the items
+//    were decoded, and issues the tile's stages with compile-time
+//    instruction descriptors: a descriptor chosen at run time slowed every
+//    tile's issue.
 //
 // Rows of the tile are assigned crosswise: the leader CTA (rank 0, whose
 // warp 1 issues the MMAs) holds tile rows [128, 256) and the peer rows
@@ -172,10 +173,10 @@ __device__ __forceinline__ Item decode_pair_item(const int64_t* plan, const int6
 __device__ __forceinline__ bool is_narrow(const Item& it) { return it.narrow != 0; }
 
 // Item w of the launch.  The plan's tiles go to the SM pairs round-robin;
-// when the last round (tiles split_from .. total - 1) would leave at least
-// half of the pairs idle, each of its tiles is dealt as two 256 x 128
-// halves instead (items split_from + 2 t and split_from + 2 t + 1), so that
-// the round takes one narrow tile's time.
+// when their last round (plan tiles split_from .. plan[batch] - 1) would
+// leave at least half of the pairs idle, each of its tiles split_from + t is
+// dealt as two 256 x 128 halves instead (items split_from + 2 t and
+// split_from + 2 t + 1), so that the round takes one narrow tile's time.
 __device__ __forceinline__ Item decode_launch_item(const int64_t* plan, const int64_t* soff, int batch, int64_t w,
                                                    int64_t chunk, int64_t split_from) {
   if (w < split_from) return decode_pair_item(plan, soff, batch, w, chunk);
