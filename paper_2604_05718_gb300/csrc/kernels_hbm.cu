@@ -209,13 +209,14 @@ __global__ void __launch_bounds__(kScanThreads) mutual_compact_kernel(int batch,
   }
   if (threadIdx.x == 0) {
     ws.count[b] = carry;
-    __threadfence();
-    const int prev = atomicAdd(reinterpret_cast<int*>(&ws.status[2]), 1);
+    // The ticket increment releases this block's count and, in the last
+    // block, acquires every other block's (their increments came first).
+    int prev;
+    asm volatile("atom.add.acq_rel.gpu.global.s32 %0, [%1], 1;" : "=r"(prev) : "l"(ws.status + 2) : "memory");
     is_last = (prev == batch - 1);
   }
   __syncthreads();
   if (!is_last) return;
-  __threadfence();
   int64_t acc = 0;
   for (int c0 = 0; c0 <= batch; c0 += kScanThreads) {
     const int idx = c0 + threadIdx.x;
