@@ -109,3 +109,14 @@ def test_all_split_fp32(mpm, pairs):
     # fp32 tokens take the three-product tf32 kernel with 8 epilogue warps.
     sizes = sizes_for(pairs // 2 - 1)
     check(mpm, sizes, 128, "f32", 73, "fp32 all split")
+
+
+def test_split_past_the_listed_items(mpm, pairs):
+    # Each pair lists its first 160 items in shared memory and decodes the
+    # rest on the fly, the narrow bit included: 161 tiles per pair and a
+    # split leftover round of pairs // 2 - 3 tiles, from images of 1 to 5
+    # tokens (one narrow tile each), on the 8-warp epilogue.
+    n_img = 161 * pairs + pairs // 2 - 3
+    rng = np.random.default_rng(74)
+    sizes = rng.integers(1, 6, n_img).tolist()
+    check(mpm, sizes, 640, "bf16", 74, f"{n_img} one-tile images")
