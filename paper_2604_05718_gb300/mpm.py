@@ -31,8 +31,8 @@ STATUS_NAMES = {
 }
 EXPORTS = ("mpm_abi_version", "mpm_status_string", "mpm_merge_workspace_size", "mpm_merge", "mpm_merge_timed",
            "mpm_compose_maps", "mpm_unmerge_gather", "mpm_nearest_neighbors", "mpm_get_device_status",
-           "mpm_merge_no_alloc", "mpm_no_alloc_get_device_status", "mpm_compose_gather", "mpm_pad_batch", "mpm_unpad_batch", "mpm_merge_chunked",
-           "mpm_nearest_neighbors_chunked")
+           "mpm_merge_no_alloc", "mpm_no_alloc_get_device_status", "mpm_compose_gather", "mpm_pad_batch",
+           "mpm_unpad_batch", "mpm_merge_chunked", "mpm_nearest_neighbors_chunked")
 
 _lib = None
 
